@@ -1,0 +1,399 @@
+"""Benchmark: decode steps over a sentinel-compressed KV cache on GB300.
+
+One step = one pass of the whole hot path over a batch: append the new token's K/V rows (all layers),
+single-query decode attention for every layer over the kept rows, and compaction of the span a <CR>
+just closed.  Workload (default): the OPT-1.3B-shaped cache (M=24, H=32, d_head=64, fp16, b=16,
+prompt 2048 with 32 of every 64 tokens enclosed, a span closed and freed every 33 generated tokens),
+seeded synthetic inputs already resident in HBM.  Every step reads ~3.1 GB, far more than L2.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl kvc|reference]
+
+Prints one JSON line (rank 0).  Multi-GPU (torchrun): every rank runs its own replica (the path
+shards by sequence with no exchange); value = tokens of all ranks / max time over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "compressed-KV decode-attention tokens/s; achieved HBM GB/s vs ~8 TB/s peak"
+UNIT = "tokens/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=128)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default="opt1.3b")
+    ap.add_argument("--impl", default="kvc", choices=["kvc", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="budget of the CPU-baseline sample")
+    return ap.parse_args()
+
+
+def measured_hbm_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            j = json.load(f)
+        return float(j["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for rel in ("paper_2310_08152_gb300/csrc/kernels.cu", "paper_2310_08152_gb300/csrc/kernels.hpp"):
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per decode launch from a committed ncu capture, if it was taken on this kernel source."""
+    p = os.path.join(ROOT, "profiles", "decode_traffic.json")
+    try:
+        with open(p) as f:
+            j = json.load(f)
+    except Exception:
+        return None
+    rec = j.get(workload)
+    if not rec or rec.get("kernel_source_hash") != kernel_source_hash():
+        return None
+    return rec.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks/throttle sampling while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------------------------
+# CPU oracle timing (the reported CPU baseline, and the reference arm)
+# ------------------------------------------------------------------------------------------------
+
+class OracleSample:
+    """Full-length masked decode of one layer for every sequence of the workload, by the fp64 oracle on
+    the host cores.  K/V of that layer are generated once for the whole capacity (not timed)."""
+
+    def __init__(self, w, steps_total: int, layer: int = 0):
+        import oracle
+        import oracle.workload as ow
+
+        self.oracle, self.ow, self.w, self.layer = oracle, ow, w, layer
+        self.K, self.V = [], []
+        for s in range(w.b):
+            T = int(w.prompt_len[s]) + steps_total
+            K, V = ow.kv_bits(w, layer, s, T)
+            self.K.append(K)
+            self.V.append(V)
+        self.threads = oracle.max_threads()
+
+    def time_step(self, g: int) -> float:
+        """Seconds the oracle takes for layer `layer` of decode step g (query = generated token g)."""
+        w, ow = self.w, self.ow
+        kinds_l, pos_l, K_l, V_l, q_l = [], [], [], [], []
+        for s in range(w.b):
+            kinds, pos = ow.history(w, s, g + 1)
+            T = kinds.size
+            kinds_l.append(kinds)
+            pos_l.append(pos)
+            K_l.append(np.ascontiguousarray(self.K[s][:, :T]))
+            V_l.append(np.ascontiguousarray(self.V[s][:, :T]))
+            q_l.append(ow.q_bits(w, self.layer, s, T - 1))
+        q = np.stack(q_l)
+        t0 = time.perf_counter()
+        self.oracle.masked_decode(kinds_l, pos_l, K_l, V_l, q, w.dtype, w.scale, rot=w.rotary_dim,
+                                  base=w.rope_base)
+        return time.perf_counter() - t0
+
+    def tokens_per_s(self, seconds_per_layer: float) -> float:
+        return self.w.b / (seconds_per_layer * self.w.M)
+
+
+def cpu_baseline(w, steps_total: int, budget_s: float):
+    samp = OracleSample(w, steps_total)
+    times = []
+    t_start = time.perf_counter()
+    g = 0
+    while True:
+        times.append(samp.time_step(g % steps_total))
+        g += 1
+        if time.perf_counter() - t_start >= budget_s or g >= steps_total:
+            break
+    per_layer = sum(times) / len(times)
+    return {"value": samp.tokens_per_s(per_layer), "unit": UNIT, "cores": samp.threads, "kind": "oracle",
+            "sample": f"fp64 oracle, full-length masked decode of layer 0 for all {w.b} sequences at {len(times)} "
+                      f"decode steps (mean {per_layer * 1e3:.1f} ms per layer), scaled by M={w.M} layers; "
+                      "K/V generation not timed"}
+
+
+# ------------------------------------------------------------------------------------------------
+# arms
+# ------------------------------------------------------------------------------------------------
+
+def dist_setup(n_gpus: int):
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != n_gpus and world > 1:
+        raise SystemExit(f"--gpus {n_gpus} but WORLD_SIZE={world}")
+    return rank, world, local
+
+
+def run_reference(args, w):
+    rank, world, _ = dist_setup(args.gpus)
+    if rank != 0:
+        return
+    steps_total = args.warmup + args.steps
+    samp = OracleSample(w, steps_total)
+    for g in range(args.warmup):
+        samp.time_step(g)
+    times = [samp.time_step(args.warmup + k) for k in range(args.steps)]
+    per_layer = sum(times) / len(times)
+    value = samp.tokens_per_s(per_layer)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_layer * w.M * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded counter-based generator)",
+        "config": workload_config(w),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": samp.threads, "kind": "oracle",
+                         "sample": f"each step: fp64 oracle full-length masked decode of layer 0 for all {w.b} "
+                                   f"sequences, scaled by M={w.M}; K/V generation not timed"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(w):
+    L = w.prompt_len
+    return {"workload": f"{w.name}: {w.note}", "M": w.M, "H": w.H, "d_head": w.d, "b": w.b,
+            "prompt_len": int(L[0]) if np.all(L == L[0]) else f"{int(L.min())}..{int(L.max())}",
+            "kv_dtype": w.dtype, "accum": "f32", "rope": bool(w.rotary_dim), "parallelism": "replicas",
+            "l2": "inputs larger than L2 (every step reads GBs of distinct K/V rows)"}
+
+
+def run_kvc(args, w):
+    import torch
+    import torch.distributed as dist
+
+    import harness
+    import paper_2310_08152_gb300 as kvc
+
+    rank, world, local = dist_setup(args.gpus)
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    steps_total = args.warmup + args.steps
+    dev = torch.device("cuda", local)
+
+    # ---------------- device-resident run ----------------
+    run = harness.Runner(w, steps_total, device=dev)
+    run.load_prompt()
+    inputs = [run.make_step_inputs(g) for g in range(steps_total)]
+    out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()
+    for g in range(args.warmup):
+        run.step(inputs[g], out)
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(w.M)]
+          for _ in range(args.steps)]
+    bytes_per_step = []
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    launches0 = run.cache.launch_count
+    clocks.start()
+    t_start.record()
+    for k in range(args.steps):
+        # decode bytes of this step are fixed once the token is appended: computed from the host lengths
+        inp = inputs[args.warmup + k]
+        run.cache.append(inp.kv_k, inp.kv_v, np.ones(w.b, np.int32), inp.kinds)
+        bytes_per_step.append(run.decode_bytes())
+        for m in range(w.M):
+            ev[k][m][0].record()
+            kvc.kvc_decode_attention(run.cache.handle, m, inp.q[m], w.scale, out[m])
+            ev[k][m][1].record()
+        seq, cl, cr = run.step_spans(inp.kinds)
+        run.g += 1
+        if seq:
+            run.cache.compress_spans(seq, cl, cr)
+    t_end.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    launches = run.cache.launch_count - launches0
+    elapsed = t_start.elapsed_time(t_end) / 1e3
+    if world > 1:
+        t = torch.tensor([elapsed], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed = float(t.item())
+    tokens = w.b * args.steps * world
+    value = tokens / elapsed
+    dec_ms = [[ev[k][m][0].elapsed_time(ev[k][m][1]) for m in range(w.M)] for k in range(args.steps)]
+    dec_total_s = sum(sum(r) for r in dec_ms) / 1e3
+    dec_bytes_total = sum(b * w.M for b in bytes_per_step)
+    achieved = dec_bytes_total / dec_total_s / 1e9
+    peak, peak_kind = measured_hbm_peak()
+    launches_decode = args.steps * w.M
+    status = run.cache.device_status()
+    del inputs, run
+    torch.cuda.empty_cache()
+
+    # ---------------- end to end through the C ABI with host buffers ----------------
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, w, dev, world)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": elapsed / args.steps * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+            "data": "synthetic (seeded counter-based generator; no dataset or weights)",
+            "config": workload_config(w),
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "peak_kind": peak_kind,
+                         "kernel": "decode_kernel (split-K single-query attention + log-sum-exp combine)",
+                         "traffic": recorded_traffic(w.name),
+                         "bytes_per_launch_mean": dec_bytes_total / launches_decode,
+                         "launch_us_mean": dec_total_s / launches_decode * 1e6},
+            "decode_share_of_step": dec_total_s / elapsed,
+            "gpu_launches": launches,
+            "device_status": status,
+            "clocks": clk,
+            "e2e": e2e,
+        }
+        if not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline(w, steps_total, args.cpu_seconds)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def run_e2e(args, w, dev, world):
+    """The same steps through the public API with inputs in pinned host memory: each step copies its
+    token's K/V and the queries host->device and reads the outputs back device->host."""
+    import torch
+    import torch.distributed as dist
+
+    import harness
+
+    steps_total = args.warmup + args.steps
+    run = harness.Runner(w, steps_total, device=dev)
+    run.load_prompt()
+    host_in = []
+    for g in range(steps_total):
+        inp = run.make_step_inputs(g)
+        host_in.append((inp.kinds, inp.kv_k.cpu().pin_memory(), inp.kv_v.cpu().pin_memory(),
+                        inp.q.cpu().pin_memory()))
+    shape = (w.M, w.b, w.H, w.d)
+    dk = torch.empty(shape, dtype=run.tdt, device=dev)
+    dv = torch.empty_like(dk)
+    dq = torch.empty_like(dk)
+    out = torch.empty(shape, dtype=torch.float32, device=dev)
+    host_out = torch.empty(shape, dtype=torch.float32).pin_memory()
+    h2d = 3 * dk.numel() * dk.element_size()
+    d2h = host_out.numel() * 4
+
+    def one(g):
+        kinds, hk, hv, hq = host_in[g]
+        dk.copy_(hk, non_blocking=True)
+        dv.copy_(hv, non_blocking=True)
+        dq.copy_(hq, non_blocking=True)
+        run.step(harness.StepInputs(kinds, dk, dv, dq), out)
+        host_out.copy_(out, non_blocking=True)
+
+    for g in range(args.warmup):
+        one(g)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for k in range(args.steps):
+        one(args.warmup + k)
+    torch.cuda.synchronize()
+    elapsed = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([elapsed], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed = float(t.item())
+    del run
+    torch.cuda.empty_cache()
+    return {"value": w.b * args.steps * world / elapsed, "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h}
+
+
+def main():
+    args = parse()
+    from synth import workloads as wl
+
+    w = wl.by_name(args.workload)
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_kvc(args, w)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,145 @@
+"""Runs a synthetic workload (synth.workloads) through the CUDA path.
+
+Shared by the GPU tests, ``__graft_entry__.smoke`` and ``bench.py``.  Inputs come
+from the device build of the seeded generator, so tens of GB of K/V never cross
+the host link.  Counter conventions (also used by the oracle side): K and V of
+history token t of sequence s use counters (i0=t, i1=s) with tag (K|V, layer);
+the query of layer m at history token t uses tag (q, m) and (i0=t, i1=s).
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import List, Optional, Tuple
+
+import numpy as np
+import torch
+
+import paper_2310_08152_gb300 as kvc
+import synth
+from synth import workloads as wl
+
+
+@dataclass
+class StepInputs:
+    kinds: np.ndarray            # [b] uint8
+    kv_k: torch.Tensor           # [M][b][H][d]
+    kv_v: torch.Tensor           # [M][b][H][d]
+    q: torch.Tensor              # [M][b][H][d]
+
+
+class Runner:
+    def __init__(self, w: wl.Workload, steps: int, policy: int = kvc.POLICY_PAPER, device=None,
+                 capacity_slack: int = 0):
+        self.w = w
+        self.steps = steps
+        self.policy = policy
+        self.device = torch.device("cuda", 0) if device is None else torch.device(device)
+        self.tdt = torch.float16 if w.dtype == "f16" else torch.bfloat16
+        cap = w.capacity(steps) + capacity_slack
+        self.cache = kvc.KVCache(w.M, w.H, w.d, cap, w.dtype, w.rotary_dim, w.rope_base, policy, device=self.device)
+        self.L = w.prompt_len.copy()
+        self.open_cl = [-1] * w.b      # history index of an open <CL>
+        self.g = 0                      # generated tokens so far
+        self.kv_scale = synth.scale_for(w.kv_sigma)
+        self.q_scale = synth.scale_for(w.q_sigma)
+
+    # ---------------------------------------------------------------------------------------
+    def _fill(self, tensor_kind: int, layer: int, tok_t: torch.Tensor, tok_s: torch.Tensor, out: torch.Tensor,
+              scale) -> torch.Tensor:
+        synth.fill_tokens_cuda(self.w.seed, self.w.dtype, scale, synth.tag(tensor_kind, layer), tok_t, tok_s,
+                               self.w.H, self.w.d, out)
+        return out
+
+    def load_prompt(self, compress: bool = True, stream=None):
+        """Append every prompt (layer by layer) and free all prompt spans in one go (Sec. 3.1)."""
+        w = self.w
+        n_new = self.L.astype(np.int32)
+        kinds = np.concatenate(w.prompt_kinds).astype(np.uint8)
+        N = int(n_new.sum())
+        tok_t = torch.from_numpy(np.concatenate([np.arange(L, dtype=np.int32) for L in self.L])).to(self.device)
+        tok_s = torch.from_numpy(np.repeat(np.arange(w.b, dtype=np.int32), self.L)).to(self.device)
+        kbuf = torch.empty(N * w.H * w.d, dtype=self.tdt, device=self.device)
+        vbuf = torch.empty_like(kbuf)
+        pos = None
+        for m in range(w.M):
+            self._fill(synth.K_TENSOR, m, tok_t, tok_s, kbuf, self.kv_scale)
+            self._fill(synth.V_TENSOR, m, tok_t, tok_s, vbuf, self.kv_scale)
+            if m == 0:
+                pos = self.cache.append(kbuf, vbuf, n_new, kinds, layer=0, stream=stream)
+            else:
+                kvc.kvc_append(self.cache.handle, m, kbuf, vbuf, None, None, None, stream)
+        del kbuf, vbuf
+        if compress:
+            self.compress_prompt(stream)
+        return pos
+
+    def compress_prompt(self, stream=None):
+        seq, cl, cr = [], [], []
+        for s in range(self.w.b):
+            for a, c in self.w.prompt_spans[s]:
+                seq.append(s)
+                cl.append(a)
+                cr.append(c)
+        if seq:
+            self.cache.compress_spans(seq, cl, cr, stream)
+
+    # ---------------------------------------------------------------------------------------
+    def make_step_inputs(self, g: int) -> StepInputs:
+        """Inputs of generated token g: its K/V rows (all layers) and the queries of all layers."""
+        w = self.w
+        kinds = np.array([w.gen_kind(s, g) for s in range(w.b)], dtype=np.uint8)
+        tok_t = torch.from_numpy((self.L + g).astype(np.int32)).to(self.device)
+        tok_s = torch.arange(w.b, dtype=torch.int32, device=self.device)
+        shape = (w.M, w.b, w.H, w.d)
+        k = torch.empty(shape, dtype=self.tdt, device=self.device)
+        v = torch.empty(shape, dtype=self.tdt, device=self.device)
+        q = torch.empty(shape, dtype=self.tdt, device=self.device)
+        for m in range(w.M):
+            self._fill(synth.K_TENSOR, m, tok_t, tok_s, k[m], self.kv_scale)
+            self._fill(synth.V_TENSOR, m, tok_t, tok_s, v[m], self.kv_scale)
+            self._fill(synth.Q_TENSOR, m, tok_t, tok_s, q[m], self.q_scale)
+        return StepInputs(kinds, k, v, q)
+
+    def step_spans(self, kinds: np.ndarray):
+        """Spans closed by this step's tokens (to free right after the step's decode)."""
+        seq, cl, cr = [], [], []
+        for s in range(self.w.b):
+            t = int(self.L[s]) + self.g
+            if kinds[s] == wl.CL:
+                self.open_cl[s] = t
+            elif kinds[s] == wl.CR:
+                seq.append(s)
+                cl.append(self.open_cl[s])
+                cr.append(t)
+                self.open_cl[s] = -1
+        return seq, cl, cr
+
+    def step(self, inp: StepInputs, out: torch.Tensor, stream=None, events=None, compress: bool = True):
+        """One decode step: append the token, decode all M layers into out[M][b][H][d], free closed spans.
+
+        events: optional list of (start, end) CUDA event pairs, one per layer, recorded around each decode."""
+        w = self.w
+        n_new = np.ones(w.b, dtype=np.int32)
+        self.cache.append(inp.kv_k, inp.kv_v, n_new, inp.kinds, layer=-1, stream=stream)
+        for m in range(w.M):
+            if events is not None:
+                events[m][0].record(stream)
+            kvc.kvc_decode_attention(self.cache.handle, m, inp.q[m], w.scale, out[m], stream)
+            if events is not None:
+                events[m][1].record(stream)
+        seq, cl, cr = self.step_spans(inp.kinds)
+        self.g += 1
+        if compress and seq:
+            self.cache.compress_spans(seq, cl, cr, stream)
+        return seq
+
+    # ---------------------------------------------------------------------------------------
+    def attended_rows(self) -> np.ndarray:
+        """Rows the next decode reads per sequence."""
+        return self.cache.lengths()[1]
+
+    def decode_bytes(self) -> int:
+        """Algorithmic bytes of one decode launch: kept K+V rows read, q read, out written."""
+        w = self.w
+        rows = int(self.attended_rows().sum())
+        return 2 * rows * w.H * w.d * 2 + w.b * w.H * w.d * 2 + w.b * w.H * w.d * 4

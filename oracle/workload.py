@@ -1,0 +1,63 @@
+"""Oracle-side regeneration of a workload's inputs and its expected decode outputs.
+
+TEST INFRASTRUCTURE ONLY (tests, smoke check, CPU baseline).  Regenerates K, V
+and q with the host build of the seeded generator, using the same counter
+conventions as the CUDA-path harness (K/V of history token t of sequence s:
+(i0=t, i1=s) with tag (K|V, layer); the query of layer m at history token t:
+tag (q, m), (i0=t, i1=s)), and runs the fp64 oracle over the FULL history under
+the mask -- never over a compacted cache.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+import synth
+from synth import workloads as wl
+
+from . import masked_decode, tied_positions, POLICY_PAPER
+
+
+def history(w: wl.Workload, s: int, steps_done: int):
+    """Kinds and positions of sequence s after the prompt and `steps_done` generated tokens."""
+    kinds = w.kinds_history(s, steps_done)
+    return kinds, tied_positions(kinds)
+
+
+def kv_bits(w: wl.Workload, layer: int, s: int, T: int, heads=None):
+    """uint16 K, V of sequence s for history tokens [0, T): shapes [len(heads), T, d]."""
+    tok_t = np.arange(T, dtype=np.int32)
+    tok_s = np.full(T, s, dtype=np.int32)
+    sc = synth.scale_for(w.kv_sigma)
+    K = synth.fill_tokens_host(w.seed, w.dtype, sc, synth.tag(synth.K_TENSOR, layer), tok_t, tok_s, w.H, w.d)
+    V = synth.fill_tokens_host(w.seed, w.dtype, sc, synth.tag(synth.V_TENSOR, layer), tok_t, tok_s, w.H, w.d)
+    K = K.transpose(1, 0, 2)
+    V = V.transpose(1, 0, 2)
+    if heads is not None:
+        K, V = K[heads], V[heads]
+    return np.ascontiguousarray(K), np.ascontiguousarray(V)
+
+
+def q_bits(w: wl.Workload, layer: int, s: int, t: int, heads=None):
+    sc = synth.scale_for(w.q_sigma)
+    q = synth.fill_tokens_host(w.seed, w.dtype, sc, synth.tag(synth.Q_TENSOR, layer), np.array([t], np.int32),
+                               np.array([s], np.int32), w.H, w.d)[0]
+    return q if heads is None else q[heads]
+
+
+def expected_decode(w: wl.Workload, steps_done: int, layer: int, seqs, heads=None, policy: int = POLICY_PAPER,
+                    n_threads: int = 0) -> np.ndarray:
+    """fp64 [len(seqs), n_heads, d]: decode of `layer` for the query at the last token of each sequence's
+    history (prompt + `steps_done` generated tokens), under the mask over the full history."""
+    kinds_l, pos_l, K_l, V_l, q_l = [], [], [], [], []
+    for s in seqs:
+        kinds, pos = history(w, s, steps_done)
+        T = kinds.size
+        K, V = kv_bits(w, layer, s, T, heads)
+        kinds_l.append(kinds)
+        pos_l.append(pos)
+        K_l.append(K)
+        V_l.append(V)
+        q_l.append(q_bits(w, layer, s, T - 1, heads))
+    q = np.stack(q_l)
+    return masked_decode(kinds_l, pos_l, K_l, V_l, q, w.dtype, w.scale, rot=w.rotary_dim, base=w.rope_base,
+                         policy=policy, n_threads=n_threads)

@@ -1,0 +1,97 @@
+// Host-side span bookkeeping of b token histories (no CUDA).
+//
+// Tracks, per sequence, the kinds and positions of every token appended so
+// far, the <CL> ... <CR> spans (Sec. 3.1: non-overlapping, paired in order),
+// which spans have been freed, and the number of stored rows.  From that it
+// derives what each device call needs: destination rows of appended tokens,
+// drop ranges of a compaction, and the rows a decode query may not see.
+#pragma once
+
+#include <cstdint>
+#include <string>
+#include <utility>
+#include <vector>
+
+namespace kvc {
+
+enum Kind : uint8_t { NORMAL = 0, CL = 1, CR = 2 };
+enum Policy : int { POLICY_PAPER = 0, POLICY_KEEP_CL = 1 };
+
+struct Span {
+  int64_t cl = -1;
+  int64_t cr = -1;  // -1 while open
+  bool freed = false;
+};
+
+// What a decode query of one sequence reads: stored rows [begin, len), except [mask_lo, mask_hi).
+struct DecodeView {
+  int64_t len = 0;
+  int64_t begin = 0;
+  int64_t mask_lo = 0;
+  int64_t mask_hi = 0;
+  int32_t qpos = 0;
+  int64_t attended() const { return len - begin - (mask_hi - mask_lo); }
+};
+
+// One sequence's part of a compaction: drop ranges in history-index space (sorted, disjoint).
+struct CompactSeq {
+  int s = 0;
+  int64_t len_old = 0;
+  int64_t len_new = 0;
+  int64_t first_row = 0;  // first stored row that is dropped
+  std::vector<std::pair<int64_t, int64_t>> drops;
+};
+
+class Book {
+ public:
+  Book(int b, Policy policy, const int64_t* capacity);
+
+  int b() const { return b_; }
+  Policy policy() const { return policy_; }
+  int64_t capacity(int s) const { return seqs_[s].cap; }
+  int64_t stored(int s) const { return seqs_[s].stored; }
+  int64_t history(int s) const { return (int64_t)seqs_[s].kind.size(); }
+
+  // Validation only (no state change).  On error returns false and sets `err`.
+  bool check_append(const int32_t* n_new, const uint8_t* kinds, std::string& err, int& code) const;
+  void next_positions(const int32_t* n_new, const uint8_t* kinds, int32_t* pos_out) const;
+  void apply_append(const int32_t* n_new, const uint8_t* kinds, const int32_t* pos);
+
+  bool plan_compress(const int32_t* seq, const int64_t* cl, const int64_t* cr, int n, std::vector<CompactSeq>& plan,
+                     std::string& err) const;
+  void apply_compress(const std::vector<CompactSeq>& plan, const int32_t* seq, const int64_t* cl, int n);
+
+  // The decode query of sequence s (its last token).  False (with `err`) if the rows hidden from it
+  // are not one contiguous run of stored rows.
+  bool decode_view(int s, DecodeView& v, std::string& err) const;
+
+  void pending_spans(int s, std::vector<std::pair<int64_t, int64_t>>& out) const;
+  // history index -> stored row (or -1 when freed)
+  int64_t stored_index(int s, int64_t j) const;
+  // visibility of every history token to the query at the last token
+  void visible(int s, uint8_t* vis) const;
+  void stored_rows(int s, std::vector<int32_t>& orig, std::vector<int32_t>& pos) const;
+  const std::vector<uint8_t>& kinds(int s) const { return seqs_[s].kind; }
+  const std::vector<int32_t>& positions(int s) const { return seqs_[s].pos; }
+
+ private:
+  struct Seq {
+    std::vector<uint8_t> kind;
+    std::vector<int32_t> pos;
+    std::vector<Span> spans;  // ordered by cl
+    int64_t normals = 0;
+    bool open = false;
+    int64_t stored = 0;
+    int64_t cap = 0;
+    std::vector<std::pair<int64_t, int64_t>> freed;  // sorted freed history ranges
+    std::vector<int64_t> freed_before;               // prefix sums of freed lengths
+  };
+  void rebuild_prefix(Seq& q);
+  int find_span(const Seq& q, int64_t cl) const;
+
+  int b_;
+  Policy policy_;
+  std::vector<Seq> seqs_;
+};
+
+}  // namespace kvc

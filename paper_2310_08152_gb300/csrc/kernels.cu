@@ -1,0 +1,848 @@
+// sm_103a kernels of the sentinel-compressed KV decode path.
+//
+//   append_kernel         new tokens' K/V rows into the ragged cache (+ RoPE on K, + metadata)
+//   compact_scan_kernel   keep flags -> warp-ballot/popc + block exclusive scan -> destination map,
+//                         in-place move of the position / history-index metadata
+//   compact_move_kernel   in-place, ascending, 16-byte vectorised row moves of every
+//                         (layer, K/V, head) stream of the affected sequences
+//   decode_kernel         split-K single-query attention over the kept rows: a producer warp streams
+//                         K/V tiles into shared memory with 1-D TMA bulk copies (cp.async.bulk +
+//                         mbarrier), eight consumer warps do fp32 dot products, warp-shuffle
+//                         reductions and an online softmax; pieces of a split row range are merged
+//                         by a log-sum-exp combine done by the last CTA to finish (arrival counter).
+//
+// No tensor cores: one query per (sequence, head) makes decode a GEMV (1 flop per byte read), far
+// below any tensor-core ridge; the kernels are bound by HBM bandwidth.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+
+#include "kernels.hpp"
+
+namespace kvc {
+namespace {
+
+constexpr unsigned kFull = 0xFFFFFFFFu;
+
+// ---------------------------------------------------------------------------------------------
+// 16-bit element types
+// ---------------------------------------------------------------------------------------------
+struct F16T {
+  static __device__ __forceinline__ float2 f2(uint32_t u) {
+    return __half22float2(*reinterpret_cast<const __half2*>(&u));
+  }
+  static __device__ __forceinline__ float f1(uint16_t u) { return __half2float(__ushort_as_half(u)); }
+  static __device__ __forceinline__ uint16_t r(float x) { return __half_as_ushort(__float2half_rn(x)); }
+};
+struct BF16T {
+  static __device__ __forceinline__ float2 f2(uint32_t u) {
+    return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u));
+  }
+  static __device__ __forceinline__ float f1(uint16_t u) { return __bfloat162float(__ushort_as_bfloat16(u)); }
+  static __device__ __forceinline__ uint16_t r(float x) { return __bfloat16_as_ushort(__float2bfloat16_rn(x)); }
+};
+
+// ---------------------------------------------------------------------------------------------
+// RoPE angle.  theta = pos * base^(-2i/rot) is reduced in turns: g = base^(-2i/rot) / (2 pi) is
+// held as a double-float (hi, lo); pos * hi is split exactly with an FMA (Dekker's two-product),
+// the integer part of the turns is removed exactly, and sincospi takes the small remainder.  The
+// angle error stays near 1e-7 rad at any position below 2^24 (a plain binary32 product would be
+// off by up to half an ulp of theta, about 5e-4 rad at position 8192).
+// ---------------------------------------------------------------------------------------------
+__device__ __forceinline__ void rope_sincos(int32_t pos, float2 g, float* s, float* c) {
+  const float p = (float)pos;
+  const float a = __fmul_rn(p, g.x);
+  const float e = __fmaf_rn(p, g.x, -a);
+  const float f = __fadd_rn(__fsub_rn(a, rintf(a)), __fmaf_rn(p, g.y, e));
+  sincospif(2.0f * f, s, c);
+}
+
+// ---------------------------------------------------------------------------------------------
+// PTX helpers: mbarrier, 1-D bulk copy (TMA), named barrier, global timer
+// ---------------------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Waits for the phase with the given parity; gives up after limit_ns (returns false).
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, unsigned long long limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 63u) == 0 && global_ns() - t0 > limit_ns) return false;
+  }
+}
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_addr(dst)),
+               "l"(src), "r"(bytes), "r"(smem_addr(bar))
+               : "memory");
+}
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// ---------------------------------------------------------------------------------------------
+// a1: append
+// ---------------------------------------------------------------------------------------------
+// Work items: [0, n_copy) copy one 16-byte vector (all of V, the unrotated columns of K);
+// [n_copy, n_copy + n_rot) rotate one pair of 8-column vectors of K for every head of one token.
+template <typename T, int D>
+__global__ void __launch_bounds__(256) append_kernel(Geometry g, Static st, Buffers buf,
+                                                     const TokPlan* __restrict__ plan, int64_t ntok, int m0,
+                                                     int n_layers, int write_meta,
+                                                     const uint16_t* __restrict__ k_in,
+                                                     const uint16_t* __restrict__ v_in) {
+  constexpr int VPR = D / 8;
+  const int H = g.H;
+  const int hv = g.rot / 16;              // vectors per rotated half
+  const int kcopy = VPR - 2 * hv;         // unrotated K vectors per row
+  const int per_row = VPR + kcopy;        // copy items per (layer, token, head)
+  const int64_t n_copy = (int64_t)n_layers * ntok * H * per_row;
+  const int64_t n_rot = (int64_t)n_layers * ntok * hv;
+  const int64_t plane = (int64_t)H * g.C;  // rows per (layer, K/V) plane
+  for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < n_copy + n_rot;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    if (idx < n_copy) {
+      const int c = (int)(idx % per_row);
+      int64_t r = idx / per_row;
+      const int h = (int)(r % H);
+      r /= H;
+      const int64_t tok = r % ntok;
+      const int l = (int)(r / ntok);
+      const TokPlan tp = plan[tok];
+      const bool is_v = c < VPR;
+      const int vec = is_v ? c : 2 * hv + (c - VPR);
+      const uint16_t* src = (is_v ? v_in : k_in) + (((int64_t)l * ntok + tok) * H + h) * D;
+      uint16_t* dst = (is_v ? buf.v : buf.k) +
+                      ((int64_t)(m0 + l) * plane + st.seq_row0[tp.s] + (int64_t)h * st.cap[tp.s] + tp.row) * D;
+      *reinterpret_cast<uint4*>(dst + vec * 8) = __ldg(reinterpret_cast<const uint4*>(src + vec * 8));
+      if (write_meta && l == 0 && h == 0 && c == 0) {
+        buf.pos[st.off[tp.s] + tp.row] = tp.pos;
+        buf.orig[st.off[tp.s] + tp.row] = tp.orig;
+      }
+    } else {
+      const int64_t w = idx - n_copy;
+      const int vec = (int)(w % hv);
+      const int64_t r = w / hv;
+      const int64_t tok = r % ntok;
+      const int l = (int)(r / ntok);
+      const TokPlan tp = plan[tok];
+      float cs[8], sn[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) rope_sincos(tp.pos, st.rope_g[vec * 8 + e], &sn[e], &cs[e]);
+      for (int h = 0; h < H; ++h) {
+        const uint16_t* src = k_in + (((int64_t)l * ntok + tok) * H + h) * D;
+        uint16_t* dst =
+            buf.k + ((int64_t)(m0 + l) * plane + st.seq_row0[tp.s] + (int64_t)h * st.cap[tp.s] + tp.row) * D;
+        uint4 a = __ldg(reinterpret_cast<const uint4*>(src + vec * 8));
+        uint4 b = __ldg(reinterpret_cast<const uint4*>(src + (vec + hv) * 8));
+        const uint16_t* xa = reinterpret_cast<const uint16_t*>(&a);
+        const uint16_t* xb = reinterpret_cast<const uint16_t*>(&b);
+        uint4 ya, yb;
+        uint16_t* pa = reinterpret_cast<uint16_t*>(&ya);
+        uint16_t* pb = reinterpret_cast<uint16_t*>(&yb);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float x1 = T::f1(xa[e]), x2 = T::f1(xb[e]);
+          pa[e] = T::r(x1 * cs[e] - x2 * sn[e]);
+          pb[e] = T::r(x2 * cs[e] + x1 * sn[e]);
+        }
+        *reinterpret_cast<uint4*>(dst + vec * 8) = ya;
+        *reinterpret_cast<uint4*>(dst + (vec + hv) * 8) = yb;
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------------------------
+// a3: keep flags + scan (one CTA per affected sequence)
+// ---------------------------------------------------------------------------------------------
+constexpr int kScanThreads = 1024;
+constexpr int kMaxSmemRanges = 1024;
+
+__device__ __forceinline__ bool in_ranges(int32_t o, const int2* rg, int nr) {
+  int a = 0, z = nr;  // first range with lo > o
+  while (a < z) {
+    const int mid = (a + z) >> 1;
+    if (rg[mid].x <= o)
+      a = mid + 1;
+    else
+      z = mid;
+  }
+  return a > 0 && o < rg[a - 1].y;
+}
+
+__global__ void __launch_bounds__(kScanThreads) compact_scan_kernel(Static st, Buffers buf,
+                                                                    const AffSeq* __restrict__ aff,
+                                                                    const int2* __restrict__ ranges,
+                                                                    int32_t* __restrict__ dst_map) {
+  __shared__ int2 srg[kMaxSmemRanges];
+  __shared__ int wsum[32];
+  __shared__ int total;
+  const AffSeq a = aff[blockIdx.x];
+  const int64_t off = st.off[a.s];
+  int32_t* pos = buf.pos + off;
+  int32_t* orig = buf.orig + off;
+  int32_t* dmap = dst_map + off;
+  const int nr = a.n_ranges;
+  const int2* rg = ranges + a.range_off;
+  if (nr <= kMaxSmemRanges) {
+    for (int i = threadIdx.x; i < nr; i += blockDim.x) srg[i] = rg[i];
+    rg = srg;
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int base = a.first_row;  // new index of the next kept row
+  for (int c0 = a.first_row; c0 < a.len_old; c0 += kScanThreads) {
+    const int i = c0 + threadIdx.x;
+    const bool valid = i < a.len_old;
+    int32_t o = 0, p = 0;
+    bool keep = false;
+    if (valid) {
+      o = orig[i];
+      p = pos[i];
+      keep = !in_ranges(o, rg, nr);
+    }
+    const unsigned bal = __ballot_sync(kFull, keep);
+    const int pre = __popc(bal & ((1u << lane) - 1u));
+    if (lane == 0) wsum[warp] = __popc(bal);
+    __syncthreads();  // also orders every read of this chunk before the writes below
+    if (warp == 0) {
+      const int v = wsum[lane];
+      int incl = v;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const int u = __shfl_up_sync(kFull, incl, d);
+        if (lane >= d) incl += u;
+      }
+      wsum[lane] = incl - v;
+      if (lane == 31) total = incl;
+    }
+    __syncthreads();
+    const int dst = base + wsum[warp] + pre;
+    if (valid) dmap[i] = keep ? dst : -1;
+    if (keep) {  // dst <= i: lands on rows already read (this chunk, after the barrier) or earlier chunks
+      orig[dst] = o;
+      pos[dst] = p;
+    }
+    base += total;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0 && base != a.len_new) atomicOr(buf.status, STATUS_CHECK);
+}
+
+// ---------------------------------------------------------------------------------------------
+// a4: row moves.  One CTA owns one (sequence, layer, K/V, head) stream and walks 128-row chunks
+// upward.  Every kept row moves down (dst < src), so stores of chunk k land below chunk k+1's
+// sources: the loads of chunk k+1 are issued before storing chunk k, and a barrier separates
+// each chunk's loads from its own stores.
+// ---------------------------------------------------------------------------------------------
+constexpr int kMoveThreads = 256;
+constexpr int kMoveRows = 128;
+
+template <int D>
+__global__ void __launch_bounds__(kMoveThreads) compact_move_kernel(Geometry g, Static st, Buffers buf,
+                                                                    const AffSeq* __restrict__ aff,
+                                                                    const int32_t* __restrict__ dst_map) {
+  constexpr int VPR = D / 8;                                  // 16-byte vectors per row
+  constexpr int U = kMoveRows * VPR / kMoveThreads;           // vectors per thread per chunk
+  static_assert(kMoveRows * VPR % kMoveThreads == 0, "chunk must split evenly");
+  const int streams = g.M * 2 * g.H;
+  const int ai = blockIdx.x / streams;
+  const int sidx = blockIdx.x % streams;
+  const int h = sidx % g.H;
+  const int kv = (sidx / g.H) & 1;
+  const int m = sidx / (2 * g.H);
+  const AffSeq a = aff[ai];
+  uint16_t* plane = kv ? buf.v : buf.k;
+  uint4* base = reinterpret_cast<uint4*>(
+      plane + ((int64_t)m * g.H * g.C + st.seq_row0[a.s] + (int64_t)h * st.cap[a.s]) * D);
+  const int32_t* dmap = dst_map + st.off[a.s];
+
+  uint4 ra[U], rb[U];
+  int da[U], db[U];
+  auto load = [&](int r0, uint4* reg, int* dv) {
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int vi = threadIdx.x + u * kMoveThreads;
+      const int row = r0 + vi / VPR;
+      const int col = vi % VPR;
+      int d = -1;
+      if (row < a.len_old) {
+        const int dr = __ldg(dmap + row);
+        if (dr >= 0) {
+          reg[u] = base[(int64_t)row * VPR + col];
+          d = dr * VPR + col;
+        }
+      }
+      dv[u] = d;
+    }
+  };
+  int r0 = a.first_row;
+  if (r0 >= a.len_old) return;
+  load(r0, ra, da);
+  for (; r0 < a.len_old; r0 += kMoveRows) {
+    const bool more = r0 + kMoveRows < a.len_old;
+    if (more) load(r0 + kMoveRows, rb, db);
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (da[u] >= 0) base[da[u]] = ra[u];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      ra[u] = rb[u];
+      da[u] = more ? db[u] : -1;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------------------------
+// a5 + a6: decode
+// ---------------------------------------------------------------------------------------------
+// Lane geometry: LPR lanes share one row; lane t reads NV vectors of VB bytes at vector indices
+// t + LPR*i.  Chosen so that the lanes of one shared-memory wavefront (8 lanes for 16-byte, 16
+// lanes for 8-byte accesses) hit distinct banks for the row size at hand.
+template <int D>
+struct Lanes {
+  static constexpr int RB = D * 2;
+  static constexpr int MODE = (RB % 128 == 0) ? 0 : ((RB % 128 == 64) ? 1 : 2);
+  static constexpr int VB = MODE == 0 ? 16 : 8;
+  static constexpr int LPR = MODE == 2 ? 4 : 8;
+  static constexpr int NV = RB / (VB * LPR);
+  static constexpr int EPV = VB / 2;
+  static constexpr int EPL = NV * EPV;
+  static constexpr int RPI = 32 / LPR;
+  static_assert(RB % 32 == 0, "d_head must be a multiple of 16");
+  static_assert(NV * VB * LPR == RB, "row must split evenly over the lanes");
+};
+
+template <int D>
+struct DecodeCfg {
+  using L = Lanes<D>;
+  static constexpr int NCW = 8;   // consumer warps
+  static constexpr int TR = 64;   // rows per tile
+  static constexpr int TILE = TR * L::RB;
+  static constexpr int S = (100 * 1024) / (2 * TILE);  // pipeline stages
+  static constexpr int KPT = TR / (NCW * L::RPI);       // rows per lane per tile
+  static constexpr int THREADS = (NCW + 1) * 32;
+  static constexpr int SMEM = 2 * S * TILE + 2 * S * 8 + 2 * NCW * D * 4 + 2 * NCW * 2 * 4;
+  static_assert(KPT >= 1 && KPT * NCW * L::RPI == TR, "tile must split evenly over the warps");
+  static_assert(S >= 2, "need at least two stages");
+};
+
+struct DecodeDev {
+  const uint16_t* k;  // layer plane
+  const uint16_t* v;
+  const DState* ds;
+  const int64_t* P;
+  int64_t R;
+  int G;
+  const uint16_t* q;
+  float* out;
+  float* partials;
+  int* counters;
+  int* status;
+  float qscale;  // scale * log2(e)
+  unsigned long long limit_ns;
+};
+
+// The sequence of tiles a CTA walks: its flat row range [lo, hi) of the concatenation over
+// (sequence, head) segments, each segment being the attended rows of one (s, h), cut into tiles of at
+// most TR rows that never cross a segment.
+struct TileIter {
+  const int64_t* P;
+  int b, H;
+  int64_t hi;
+  int s, h;
+  int64_t Lc, r, x;
+  __device__ void init(const int64_t* P_, int b_, int H_, int64_t lo, int64_t hi_) {
+    P = P_;
+    b = b_;
+    H = H_;
+    hi = hi_;
+    int a = 0, z = b - 1;  // largest s with H * P[s] <= lo
+    while (a < z) {
+      const int mid = (a + z + 1) >> 1;
+      if ((int64_t)H * P[mid] <= lo)
+        a = mid;
+      else
+        z = mid - 1;
+    }
+    s = a;
+    Lc = P[s + 1] - P[s];
+    const int64_t o = lo - (int64_t)H * P[s];
+    h = (int)(o / Lc);
+    r = o % Lc;
+    x = lo;
+  }
+  __device__ bool done() const { return x >= hi; }
+  __device__ int n(int TR) const {
+    int64_t k = Lc - r;
+    if (hi - x < k) k = hi - x;
+    return (int)(k < TR ? k : TR);
+  }
+  __device__ void advance(int n) {
+    x += n;
+    r += n;
+    if (r == Lc && x < hi) {
+      r = 0;
+      if (++h == H) {
+        h = 0;
+        do {
+          ++s;
+        } while (P[s + 1] == P[s]);
+        Lc = P[s + 1] - P[s];
+      }
+    }
+  }
+};
+
+__device__ __forceinline__ int cta_of(int64_t x, int64_t R, int G) { return (int)(((x + 1) * G - 1) / R); }
+
+template <typename T, int D>
+__global__ void __launch_bounds__(DecodeCfg<D>::THREADS, 2)
+    decode_kernel(Geometry g, Static st, DecodeDev p) {
+  using C = DecodeCfg<D>;
+  using L = Lanes<D>;
+  extern __shared__ __align__(128) unsigned char smem[];
+  unsigned char* sK = smem;
+  unsigned char* sV = smem + C::S * C::TILE;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + 2 * C::S * C::TILE);
+  uint64_t* empty = full + C::S;
+  float* mo = reinterpret_cast<float*>(empty + C::S);  // [2][NCW][D]
+  float* mml = mo + 2 * C::NCW * D;                     // [2][NCW][2]
+
+  const int cta = blockIdx.x;
+  const int64_t lo = (int64_t)cta * p.R / p.G;
+  const int64_t hi = (int64_t)(cta + 1) * p.R / p.G;
+  if (lo >= hi) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+#pragma unroll
+    for (int i = 0; i < C::S; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], C::NCW);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  TileIter it;
+  it.init(p.P, g.b, g.H, lo, hi);
+
+  if (warp == C::NCW) {
+    // ------------------------------- producer -------------------------------
+    if (lane != 0) return;
+    int t = 0;
+    bool ok = true;
+    int cur_s = -1;
+    int64_t seg_base = 0;
+    while (!it.done()) {
+      const int n = it.n(C::TR);
+      const int stage = t % C::S;
+      if (t >= C::S && !mbar_wait_bounded(&empty[stage], ((t / C::S) - 1) & 1, p.limit_ns)) {
+        ok = false;
+        break;
+      }
+      if (it.s != cur_s) {
+        cur_s = it.s;
+        seg_base = st.seq_row0[cur_s] + p.ds[cur_s].begin;
+      }
+      const int64_t row = seg_base + (int64_t)it.h * st.cap[cur_s] + it.r;
+      const uint32_t bytes = (uint32_t)n * L::RB;
+      mbar_arrive_expect_tx(&full[stage], 2 * bytes);
+      bulk_g2s(sK + stage * C::TILE, p.k + row * D, bytes, &full[stage]);
+      bulk_g2s(sV + stage * C::TILE, p.v + row * D, bytes, &full[stage]);
+      it.advance(n);
+      ++t;
+    }
+    if (!ok) atomicOr(p.status, STATUS_TIMEOUT);
+    // never leave with copies in flight into this CTA's shared memory
+    for (int u = t - C::S < 0 ? 0 : t - C::S; u < t; ++u) mbar_wait_bounded(&full[u % C::S], (u / C::S) & 1, p.limit_ns);
+    return;
+  }
+
+  // ------------------------------- consumers -------------------------------
+  const int grp = lane / L::LPR;  // row group within the warp
+  const int tl = lane % L::LPR;   // position within the row
+  float qv[L::EPL], o[L::EPL];
+  float m = -INFINITY, l = 0.f;
+  int64_t mask_lo = 0, mask_hi = 0, begin = 0;
+  int cur_s = -1;
+  bool dead = false;  // a bounded wait ran out: keep walking (barriers stay matched) but write nothing
+  bool piece_start = true, piece_whole = false;
+  int piece = 0;
+  int t = 0;
+  while (!it.done()) {
+    const int s = it.s, h = it.h;
+    const int64_t r0 = it.r;
+    const int n = it.n(C::TR);
+    const int stage = t % C::S;
+    if (piece_start) {
+      if (s != cur_s) {
+        cur_s = s;
+        const DState d = p.ds[s];
+        mask_lo = d.mask_lo;
+        mask_hi = d.mask_hi;
+        begin = d.begin;
+      }
+      const uint16_t* qrow = p.q + ((int64_t)s * g.H + h) * D;
+      const int32_t qpos = p.ds[s].qpos;
+      const int half = g.rot / 2;
+#pragma unroll
+      for (int i = 0; i < L::NV; ++i) {
+#pragma unroll
+        for (int e = 0; e < L::EPV; ++e) {
+          const int c = (tl + L::LPR * i) * L::EPV + e;
+          float x = T::f1(qrow[c]);
+          if (c < g.rot) {
+            const bool lo_half = c < half;
+            const float y = T::f1(qrow[lo_half ? c + half : c - half]);
+            float sn, cs;
+            rope_sincos(qpos, st.rope_g[lo_half ? c : c - half], &sn, &cs);
+            x = lo_half ? x * cs - y * sn : x * cs + y * sn;
+          }
+          qv[i * L::EPV + e] = x * p.qscale;
+          o[i * L::EPV + e] = 0.f;
+        }
+      }
+      m = -INFINITY;
+      l = 0.f;
+      piece_whole = (r0 == 0);
+      piece_start = false;
+    }
+    if (!dead && !mbar_wait_bounded(&full[stage], (t / C::S) & 1, p.limit_ns)) {
+      dead = true;
+      if (lane == 0) atomicOr(p.status, STATUS_TIMEOUT);
+    }
+    if (!dead) {
+      const unsigned char* kt = sK + stage * C::TILE;
+      const unsigned char* vt = sV + stage * C::TILE;
+      float z[C::KPT];
+#pragma unroll
+      for (int k = 0; k < C::KPT; ++k) {
+        const int j = (k * C::NCW + warp) * L::RPI + grp;
+        float acc = 0.f;
+#pragma unroll
+        for (int i = 0; i < L::NV; ++i) {
+          const unsigned char* ptr = kt + j * L::RB + (tl + L::LPR * i) * L::VB;
+          uint32_t w[L::VB / 4];
+          if constexpr (L::VB == 16) {
+            const uint4 u = *reinterpret_cast<const uint4*>(ptr);
+            w[0] = u.x;
+            w[1] = u.y;
+            w[2] = u.z;
+            w[3] = u.w;
+          } else {
+            const uint2 u = *reinterpret_cast<const uint2*>(ptr);
+            w[0] = u.x;
+            w[1] = u.y;
+          }
+#pragma unroll
+          for (int q2 = 0; q2 < L::VB / 4; ++q2) {
+            const float2 f = T::f2(w[q2]);
+            acc = fmaf(qv[i * L::EPV + 2 * q2], f.x, acc);
+            acc = fmaf(qv[i * L::EPV + 2 * q2 + 1], f.y, acc);
+          }
+        }
+#pragma unroll
+        for (int off = L::LPR / 2; off >= 1; off >>= 1) acc += __shfl_xor_sync(kFull, acc, off);
+        const int64_t row = begin + r0 + j;
+        const bool valid = j < n && !(row >= mask_lo && row < mask_hi);
+        z[k] = valid ? acc : -INFINITY;
+      }
+      float mt = z[0];
+#pragma unroll
+      for (int k = 1; k < C::KPT; ++k) mt = fmaxf(mt, z[k]);
+      const float mn = fmaxf(m, mt);
+      const float alpha = (mn == -INFINITY) ? 1.f : exp2f(m - mn);
+      l *= alpha;
+#pragma unroll
+      for (int e = 0; e < L::EPL; ++e) o[e] *= alpha;
+#pragma unroll
+      for (int k = 0; k < C::KPT; ++k) {
+        if (z[k] != -INFINITY) {
+          const int j = (k * C::NCW + warp) * L::RPI + grp;
+          const float pk = exp2f(z[k] - mn);
+          l += pk;
+#pragma unroll
+          for (int i = 0; i < L::NV; ++i) {
+            const unsigned char* ptr = vt + j * L::RB + (tl + L::LPR * i) * L::VB;
+            uint32_t w[L::VB / 4];
+            if constexpr (L::VB == 16) {
+              const uint4 u = *reinterpret_cast<const uint4*>(ptr);
+              w[0] = u.x;
+              w[1] = u.y;
+              w[2] = u.z;
+              w[3] = u.w;
+            } else {
+              const uint2 u = *reinterpret_cast<const uint2*>(ptr);
+              w[0] = u.x;
+              w[1] = u.y;
+            }
+#pragma unroll
+            for (int q2 = 0; q2 < L::VB / 4; ++q2) {
+              const float2 f = T::f2(w[q2]);
+              o[i * L::EPV + 2 * q2] = fmaf(pk, f.x, o[i * L::EPV + 2 * q2]);
+              o[i * L::EPV + 2 * q2 + 1] = fmaf(pk, f.y, o[i * L::EPV + 2 * q2 + 1]);
+            }
+          }
+        }
+      }
+      m = mn;
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[stage]);
+    const bool seg_done = (r0 + n == it.Lc);
+    it.advance(n);
+    ++t;
+    if (!(seg_done || it.done())) continue;
+
+    // --------------------------- piece end: merge ---------------------------
+#pragma unroll
+    for (int off = L::LPR; off < 32; off <<= 1) {
+      const float m2 = __shfl_xor_sync(kFull, m, off);
+      const float l2 = __shfl_xor_sync(kFull, l, off);
+      const float mn = fmaxf(m, m2);
+      const float a1 = (m == -INFINITY) ? 0.f : exp2f(m - mn);
+      const float a2 = (m2 == -INFINITY) ? 0.f : exp2f(m2 - mn);
+      l = l * a1 + l2 * a2;
+#pragma unroll
+      for (int e = 0; e < L::EPL; ++e) o[e] = o[e] * a1 + __shfl_xor_sync(kFull, o[e], off) * a2;
+      m = mn;
+    }
+    const int bsel = piece & 1;
+    float* mo_b = mo + bsel * C::NCW * D;
+    float* ml_b = mml + bsel * C::NCW * 2;
+    if (grp == 0) {
+#pragma unroll
+      for (int i = 0; i < L::NV; ++i)
+#pragma unroll
+        for (int e = 0; e < L::EPV; ++e) mo_b[warp * D + (tl + L::LPR * i) * L::EPV + e] = o[i * L::EPV + e];
+    }
+    if (lane == 0) {
+      ml_b[warp * 2] = m;
+      ml_b[warp * 2 + 1] = l;
+    }
+    named_bar_sync(1, C::NCW * 32);
+    if (warp == 0 && !dead) {
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < C::NCW; ++w) M = fmaxf(M, ml_b[w * 2]);
+      float ew[C::NCW];
+      float Lsum = 0.f;
+#pragma unroll
+      for (int w = 0; w < C::NCW; ++w) {
+        const float mw = ml_b[w * 2];
+        ew[w] = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
+        Lsum += ml_b[w * 2 + 1] * ew[w];
+      }
+      const int seg = s * g.H + h;
+      if (piece_whole && seg_done) {
+        const float inv = 1.f / Lsum;
+        for (int col = lane; col < D; col += 32) {
+          float O = 0.f;
+#pragma unroll
+          for (int w = 0; w < C::NCW; ++w) O += mo_b[w * D + col] * ew[w];
+          p.out[(int64_t)seg * D + col] = O * inv;
+        }
+      } else {
+        float* pp = p.partials + (int64_t)(cta + seg) * (D + 4);
+        for (int col = lane; col < D; col += 32) {
+          float O = 0.f;
+#pragma unroll
+          for (int w = 0; w < C::NCW; ++w) O += mo_b[w * D + col] * ew[w];
+          pp[4 + col] = O;
+        }
+        if (lane == 0) {
+          pp[0] = M;
+          pp[1] = Lsum;
+        }
+        __threadfence();
+        __syncwarp();
+        const int64_t Lc = p.P[s + 1] - p.P[s];
+        const int64_t A = (int64_t)g.H * p.P[s] + (int64_t)h * Lc;
+        const int c_first = cta_of(A, p.R, p.G);
+        const int c_last = cta_of(A + Lc - 1, p.R, p.G);
+        int last = 0;
+        if (lane == 0) last = atomicAdd(&p.counters[seg], 1) == (c_last - c_first);
+        last = __shfl_sync(kFull, last, 0);
+        if (last) {
+          __threadfence();
+          float Mx = -INFINITY;
+          for (int c = c_first; c <= c_last; ++c) Mx = fmaxf(Mx, __ldcg(p.partials + (int64_t)(c + seg) * (D + 4)));
+          float Lx = 0.f;
+          for (int c = c_first; c <= c_last; ++c) {
+            const float* q = p.partials + (int64_t)(c + seg) * (D + 4);
+            const float mc = __ldcg(q);
+            Lx += (mc == -INFINITY) ? 0.f : __ldcg(q + 1) * exp2f(mc - Mx);
+          }
+          const float inv = 1.f / Lx;
+          for (int col = lane; col < D; col += 32) {
+            float O = 0.f;
+            for (int c = c_first; c <= c_last; ++c) {
+              const float* q = p.partials + (int64_t)(c + seg) * (D + 4);
+              const float mc = __ldcg(q);
+              if (mc != -INFINITY) O += __ldcg(q + 4 + col) * exp2f(mc - Mx);
+            }
+            p.out[(int64_t)seg * D + col] = O * inv;
+          }
+          if (lane == 0) p.counters[seg] = 0;
+        }
+      }
+    }
+    ++piece;
+    piece_start = true;
+  }
+}
+
+// ---------------------------------------------------------------------------------------------
+// dispatch
+// ---------------------------------------------------------------------------------------------
+template <typename T, int D>
+cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a, int num_sms,
+                            cudaStream_t stream, int* grid) {
+  using C = DecodeCfg<D>;
+  static int occ = -1;
+  if (occ < 0) {
+    cudaError_t e = cudaFuncSetAttribute(decode_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    int o = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, decode_kernel<T, D>, C::THREADS, C::SMEM);
+    if (e != cudaSuccess) return e;
+    occ = o < 1 ? 1 : o;
+  }
+  int64_t G = (int64_t)occ * num_sms;
+  const int64_t by_work = (a.R + 2 * C::TR - 1) / (2 * C::TR);
+  if (by_work < G) G = by_work;
+  if (G > kMaxDecodeCtas) G = kMaxDecodeCtas;
+  if (G < 1) G = 1;
+  DecodeDev p;
+  const int64_t plane = (int64_t)g.H * g.C * D;
+  p.k = buf.k + (int64_t)a.layer * plane;
+  p.v = buf.v + (int64_t)a.layer * plane;
+  p.ds = a.dstate;
+  p.P = a.P;
+  p.R = a.R;
+  p.G = (int)G;
+  p.q = static_cast<const uint16_t*>(a.q);
+  p.out = a.out;
+  p.partials = a.partials;
+  p.counters = a.counters;
+  p.status = buf.status;
+  p.qscale = a.scale * 1.4426950408889634f;
+  p.limit_ns = a.wait_limit_ns;
+  decode_kernel<T, D><<<(unsigned)G, C::THREADS, C::SMEM, stream>>>(g, st, p);
+  *grid = (int)G;
+  return cudaGetLastError();
+}
+
+template <typename T, int D>
+cudaError_t launch_append_t(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t ntok,
+                            int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
+                            cudaStream_t stream) {
+  constexpr int VPR = D / 8;
+  const int hv = g.rot / 16;
+  const int64_t n_items =
+      (int64_t)n_layers * ntok * ((int64_t)g.H * (VPR + VPR - 2 * hv) + hv);
+  int64_t blocks = (n_items + 255) / 256;
+  if (blocks > 65535LL * 16) blocks = 65535LL * 16;
+  if (blocks < 1) blocks = 1;
+  append_kernel<T, D><<<(unsigned)blocks, 256, 0, stream>>>(g, st, buf, plan, ntok, m0, n_layers, write_meta ? 1 : 0,
+                                                            static_cast<const uint16_t*>(k_in),
+                                                            static_cast<const uint16_t*>(v_in));
+  return cudaGetLastError();
+}
+
+template <typename F>
+cudaError_t by_dhead(int D, F&& f) {
+  switch (D) {
+    case 64:
+      return f(std::integral_constant<int, 64>{});
+    case 80:
+      return f(std::integral_constant<int, 80>{});
+    case 96:
+      return f(std::integral_constant<int, 96>{});
+    case 128:
+      return f(std::integral_constant<int, 128>{});
+    default:
+      return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+
+bool dhead_supported(int D) { return D == 64 || D == 80 || D == 96 || D == 128; }
+
+cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t ntok,
+                          int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
+                          cudaStream_t stream) {
+  return by_dhead(g.D, [&](auto dc) {
+    constexpr int D = decltype(dc)::value;
+    if (g.dtype == 1) return launch_append_t<BF16T, D>(g, st, buf, plan, ntok, m0, n_layers, write_meta, k_in, v_in, stream);
+    return launch_append_t<F16T, D>(g, st, buf, plan, ntok, m0, n_layers, write_meta, k_in, v_in, stream);
+  });
+}
+
+cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& buf, const AffSeq* aff, int n_aff,
+                           const int32_t* ranges, int32_t* dst_map, cudaStream_t stream, int* launched) {
+  *launched = 0;
+  if (n_aff <= 0) return cudaSuccess;
+  compact_scan_kernel<<<n_aff, kScanThreads, 0, stream>>>(st, buf, aff, reinterpret_cast<const int2*>(ranges),
+                                                         dst_map);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  *launched = 1;
+  const int64_t blocks = (int64_t)n_aff * g.M * 2 * g.H;
+  e = by_dhead(g.D, [&](auto dc) {
+    constexpr int D = decltype(dc)::value;
+    compact_move_kernel<D><<<(unsigned)blocks, kMoveThreads, 0, stream>>>(g, st, buf, aff, dst_map);
+    return cudaGetLastError();
+  });
+  if (e == cudaSuccess) *launched = 2;
+  return e;
+}
+
+cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a, int num_sms,
+                          cudaStream_t stream, int* grid) {
+  *grid = 0;
+  if (a.R <= 0) return cudaSuccess;
+  return by_dhead(g.D, [&](auto dc) {
+    constexpr int D = decltype(dc)::value;
+    if (g.dtype == 1) return launch_decode_t<BF16T, D>(g, st, buf, a, num_sms, stream, grid);
+    return launch_decode_t<F16T, D>(g, st, buf, a, num_sms, stream, grid);
+  });
+}
+
+}  // namespace kvc

@@ -1,0 +1,81 @@
+// Internal interface between the host state (kvc.cpp) and the sm_103a kernels (kernels.cu).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+namespace kvc {
+
+// Per-sequence decode state, uploaded after every change of the span book.
+// The decode query of sequence s reads stored rows [begin, len) except [mask_lo, mask_hi).
+struct DState {
+  int32_t len, begin, mask_lo, mask_hi, qpos, pad0, pad1, pad2;
+};
+
+// One appended token: its sequence, destination row, position and history index.
+struct TokPlan {
+  int32_t s, row, pos, orig;
+};
+
+// One sequence of a compaction; its drop ranges (history indices, [lo, hi)) are
+// ranges[range_off .. range_off + n_ranges).
+struct AffSeq {
+  int32_t s, len_old, len_new, first_row, range_off, n_ranges, pad0, pad1;
+};
+
+// Status word bits written by kernels.
+enum : int { STATUS_TIMEOUT = 1, STATUS_CHECK = 2 };
+
+struct Geometry {
+  int M, H, D, b;
+  int64_t C;  // sum of capacities (rows per (layer, K/V, head) plane)
+  int dtype;  // 0 f16, 1 bf16
+  int rot;    // rotary dims (0 = none)
+};
+
+struct Static {
+  const int64_t* seq_row0;  // [b] H * off[s]
+  const int32_t* cap;       // [b]
+  const int64_t* off;       // [b]
+  const float2* rope_g;     // [rot/2] theta_i / (2 pi) per position as a double-float (hi, lo)
+};
+
+struct Buffers {
+  uint16_t* k;   // cache K base
+  uint16_t* v;   // cache V base
+  int32_t* pos;  // [C]
+  int32_t* orig; // [C]
+  int* status;
+};
+
+// Largest decode grid; sizes the split-K partial buffer.
+constexpr int kMaxDecodeCtas = 4096;
+
+bool dhead_supported(int D);
+
+cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t ntok,
+                          int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
+                          cudaStream_t stream);
+
+cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& buf, const AffSeq* aff, int n_aff,
+                           const int32_t* ranges, int32_t* dst_map, cudaStream_t stream, int* launched);
+
+struct DecodeArgs {
+  int layer;
+  const DState* dstate;  // [b]
+  const int64_t* P;      // [b+1] prefix sums of attended-range lengths (len - begin)
+  int64_t R;             // H * P[b]
+  const void* q;         // [b][H][D]
+  float* out;            // [b][H][D]
+  float scale;
+  float* partials;       // [(kMaxDecodeCtas + b*H) * (D + 4)]
+  int* counters;         // [b*H], zero between launches
+  unsigned long long wait_limit_ns;
+};
+
+// Returns the grid used through *grid (0 if nothing launched).
+cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a,
+                          int num_sms, cudaStream_t stream, int* grid);
+
+}  // namespace kvc

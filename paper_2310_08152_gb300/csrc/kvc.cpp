@@ -1,0 +1,702 @@
+// C ABI of the sentinel-compressed KV cache (declared in include/kvc.h): argument checks, the span
+// book, staging of per-call plans to the device, and kernel launches.
+#include "kvc.h"
+
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <deque>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "book.hpp"
+#include "kernels.hpp"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+kvc_status fail(kvc_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  std::vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+kvc_status ok() {
+  g_last_error.clear();
+  return KVC_OK;
+}
+
+kvc_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(KVC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+constexpr double kPi = 3.14159265358979323846;
+
+size_t align_up(size_t n, size_t a) { return (n + a - 1) / a * a; }
+
+// Byte offsets of the workspace regions.
+struct WsLayout {
+  size_t hdr = 0;        // int status word
+  size_t st_row0 = 0;    // int64 [b]
+  size_t st_cap = 0;     // int32 [b]
+  size_t st_off = 0;     // int64 [b]
+  size_t st_rope = 0;    // float2 [max(1, rot/2)]
+  size_t dyn = 0;        // [DState b][int64 P b+1][payload]
+  size_t dyn_P = 0;      // offset of P inside dyn
+  size_t dyn_payload = 0;  // offset of the payload inside dyn
+  size_t dyn_bytes = 0;
+  size_t dst_map = 0;    // int32 [C]
+  size_t counters = 0;   // int32 [b*H]
+  size_t partials = 0;   // float [(kMaxDecodeCtas + b*H) * (D + 4)]
+  size_t total = 0;
+};
+
+WsLayout ws_layout(int b, int H, int D, int rot, int64_t C) {
+  WsLayout L;
+  size_t o = 0;
+  auto take = [&](size_t n) {
+    size_t r = o;
+    o += align_up(n, 256);
+    return r;
+  };
+  L.hdr = take(256);
+  L.st_row0 = take(8 * (size_t)b);
+  L.st_cap = take(4 * (size_t)b);
+  L.st_off = take(8 * (size_t)b);
+  L.st_rope = take(8 * (size_t)std::max(1, rot / 2));
+  L.dyn_P = align_up(sizeof(kvc::DState) * (size_t)b, 16);
+  L.dyn_payload = align_up(L.dyn_P + 8 * (size_t)(b + 1), 16);
+  const size_t tok = sizeof(kvc::TokPlan) * (size_t)C;
+  const size_t cmp = sizeof(kvc::AffSeq) * (size_t)b + 8 * (size_t)(C / 2 + 1);
+  L.dyn_bytes = L.dyn_payload + std::max(tok, cmp);
+  L.dyn = take(L.dyn_bytes);
+  L.dst_map = take(4 * (size_t)C);
+  L.counters = take(4 * (size_t)b * H);
+  L.partials = take(4 * (size_t)(kvc::kMaxDecodeCtas + (int64_t)b * H) * (size_t)(D + 4));
+  L.total = o;
+  return L;
+}
+
+kvc_status check_config(const kvc_config* c, int64_t* C_out) {
+  if (!c) return fail(KVC_ERR_INVALID_ARG, "config is NULL");
+  if (c->M <= 0 || c->H <= 0 || c->b <= 0)
+    return fail(KVC_ERR_INVALID_ARG, "M=%d, H=%d, b=%d must be positive", c->M, c->H, c->b);
+  if (!kvc::dhead_supported(c->d_head))
+    return fail(KVC_ERR_UNSUPPORTED, "d_head=%d is not built (64, 80, 96, 128)", c->d_head);
+  if (c->dtype != KVC_F16 && c->dtype != KVC_BF16) return fail(KVC_ERR_UNSUPPORTED, "dtype %d", c->dtype);
+  if (c->rotary_dim < 0 || c->rotary_dim > c->d_head || c->rotary_dim % 16 != 0)
+    return fail(KVC_ERR_UNSUPPORTED, "rotary_dim=%d must be a multiple of 16 in [0, d_head]", c->rotary_dim);
+  if (c->rotary_dim > 0 && !(c->rope_base > 1.0f))
+    return fail(KVC_ERR_INVALID_ARG, "rope_base=%g must exceed 1", (double)c->rope_base);
+  if (c->policy != KVC_POLICY_PAPER && c->policy != KVC_POLICY_KEEP_CL)
+    return fail(KVC_ERR_INVALID_ARG, "policy %d", (int)c->policy);
+  if (!c->seq_capacity) return fail(KVC_ERR_INVALID_ARG, "seq_capacity is NULL");
+  int64_t C = 0;
+  for (int s = 0; s < c->b; ++s) {
+    if (c->seq_capacity[s] < 1 || c->seq_capacity[s] >= INT32_MAX)
+      return fail(KVC_ERR_INVALID_ARG, "seq_capacity[%d]=%lld out of range", s, (long long)c->seq_capacity[s]);
+    C += c->seq_capacity[s];
+  }
+  if ((int64_t)c->H * C >= ((int64_t)1 << 40)) return fail(KVC_ERR_INVALID_ARG, "cache too large");
+  if (C >= INT32_MAX) return fail(KVC_ERR_INVALID_ARG, "sum of capacities must stay below 2^31");
+  *C_out = C;
+  return KVC_OK;
+}
+
+// Pinned host staging ring: each upload reserves a slot, fills it, enqueues one H2D copy and
+// records an event; a slot is reused only after its copy completed.
+class PinnedRing {
+ public:
+  ~PinnedRing() { release(); }
+  cudaError_t init(size_t bytes) {
+    cap_ = align_up(bytes, 256);
+    return cudaHostAlloc(reinterpret_cast<void**>(&base_), cap_, cudaHostAllocDefault);
+  }
+  void release() {
+    for (auto& p : pending_) cudaEventDestroy(p.ev);
+    for (auto e : free_) cudaEventDestroy(e);
+    pending_.clear();
+    free_.clear();
+    if (base_) cudaFreeHost(base_);
+    base_ = nullptr;
+  }
+  // Returns nullptr if n exceeds the ring or a wait failed.
+  unsigned char* reserve(size_t n, cudaError_t* err) {
+    n = align_up(n, 256);
+    *err = cudaSuccess;
+    if (n > cap_) return nullptr;
+    if (head_ + n > cap_) head_ = 0;
+    for (auto it = pending_.begin(); it != pending_.end();) {
+      if (it->off < head_ + n && head_ < it->off + it->len) {
+        cudaError_t e = cudaEventSynchronize(it->ev);
+        if (e != cudaSuccess) {
+          *err = e;
+          return nullptr;
+        }
+        free_.push_back(it->ev);
+        it = pending_.erase(it);
+      } else {
+        ++it;
+      }
+    }
+    res_ = n;
+    return base_ + head_;
+  }
+  cudaError_t commit(void* dev_dst, size_t bytes, cudaStream_t stream) {
+    cudaError_t e = cudaMemcpyAsync(dev_dst, base_ + head_, bytes, cudaMemcpyHostToDevice, stream);
+    if (e != cudaSuccess) return e;
+    cudaEvent_t ev;
+    if (!free_.empty()) {
+      ev = free_.back();
+      free_.pop_back();
+    } else {
+      e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+      if (e != cudaSuccess) return e;
+    }
+    e = cudaEventRecord(ev, stream);
+    if (e != cudaSuccess) return e;
+    pending_.push_back({head_, res_, ev});
+    head_ += res_;
+    return cudaSuccess;
+  }
+
+ private:
+  struct Pending {
+    size_t off, len;
+    cudaEvent_t ev;
+  };
+  unsigned char* base_ = nullptr;
+  size_t cap_ = 0, head_ = 0, res_ = 0;
+  std::deque<Pending> pending_;
+  std::vector<cudaEvent_t> free_;
+};
+
+}  // namespace
+
+struct kvc_book {
+  kvc::Book book;
+  kvc_book(int b, kvc::Policy p, const int64_t* cap) : book(b, p, cap) {}
+};
+
+struct kvc_cache {
+  kvc_config cfg{};
+  std::vector<int64_t> cap, off;
+  int64_t C = 0;
+  kvc_book bk;
+  WsLayout ws;
+  // device binding (first call with a stream)
+  bool cuda_ready = false;
+  int device = -1;
+  int num_sms = 0;
+  PinnedRing ring;
+  // token batch in progress: layers [0, layers_done) written
+  int layers_done = 0;
+  int64_t batch_ntok = 0;
+  // decode readiness of the uploaded state
+  bool decode_ok = false;
+  std::string decode_err;
+  int64_t R = 0;
+  int64_t launches = 0;
+
+  kvc_cache(const kvc_config& c, int64_t C_) : cfg(c), C(C_), bk(c.b, (kvc::Policy)c.policy, c.seq_capacity) {
+    cap.assign(c.seq_capacity, c.seq_capacity + c.b);
+    off.resize(c.b);
+    int64_t o = 0;
+    for (int s = 0; s < c.b; ++s) {
+      off[s] = o;
+      o += cap[s];
+    }
+    ws = ws_layout(c.b, c.H, c.d_head, c.rotary_dim, C);
+    layers_done = c.M;
+  }
+
+  unsigned char* wsp(size_t o) const { return static_cast<unsigned char*>(cfg.workspace) + o; }
+
+  kvc::Geometry geom() const {
+    kvc::Geometry g;
+    g.M = cfg.M;
+    g.H = cfg.H;
+    g.D = cfg.d_head;
+    g.b = cfg.b;
+    g.C = C;
+    g.dtype = cfg.dtype;
+    g.rot = cfg.rotary_dim;
+    return g;
+  }
+  kvc::Static stat() const {
+    kvc::Static s;
+    s.seq_row0 = reinterpret_cast<const int64_t*>(wsp(ws.st_row0));
+    s.cap = reinterpret_cast<const int32_t*>(wsp(ws.st_cap));
+    s.off = reinterpret_cast<const int64_t*>(wsp(ws.st_off));
+    s.rope_g = reinterpret_cast<const float2*>(wsp(ws.st_rope));
+    return s;
+  }
+  kvc::Buffers bufs() const {
+    kvc::Buffers b;
+    b.k = static_cast<uint16_t*>(cfg.k_base);
+    b.v = static_cast<uint16_t*>(cfg.v_base);
+    b.pos = cfg.pos_base;
+    b.orig = cfg.orig_base;
+    b.status = reinterpret_cast<int*>(wsp(ws.hdr));
+    return b;
+  }
+
+  kvc_status ensure_cuda(cudaStream_t stream) {
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (cuda_ready) {
+      if (dev != device) return fail(KVC_ERR_STATE, "cache is bound to device %d but device %d is current", device, dev);
+      return KVC_OK;
+    }
+    e = cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    e = ring.init(2 * ws.dyn_bytes + 2 * ws.st_rope + 65536);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaHostAlloc (staging ring)");
+    // static tables
+    const int b = cfg.b, half = std::max(1, cfg.rotary_dim / 2);
+    const size_t st_bytes = ws.st_rope + 8 * (size_t)half - ws.st_row0;
+    unsigned char* h = ring.reserve(st_bytes, &e);
+    if (!h) return e != cudaSuccess ? cuda_fail(e, "staging") : fail(KVC_ERR_INVALID_ARG, "static tables exceed ring");
+    std::memset(h, 0, st_bytes);
+    int64_t* row0 = reinterpret_cast<int64_t*>(h + (ws.st_row0 - ws.st_row0));
+    int32_t* capd = reinterpret_cast<int32_t*>(h + (ws.st_cap - ws.st_row0));
+    int64_t* offd = reinterpret_cast<int64_t*>(h + (ws.st_off - ws.st_row0));
+    float* rope = reinterpret_cast<float*>(h + (ws.st_rope - ws.st_row0));
+    for (int s = 0; s < b; ++s) {
+      row0[s] = (int64_t)cfg.H * off[s];
+      capd[s] = (int32_t)cap[s];
+      offd[s] = off[s];
+    }
+    // theta_i / (2 pi) per unit position, i < rot/2, as a double-float pair
+    for (int i = 0; i < cfg.rotary_dim / 2; ++i) {
+      const double g = std::pow((double)cfg.rope_base, -2.0 * i / (double)cfg.rotary_dim) / (2.0 * kPi);
+      const float hi = (float)g;
+      rope[2 * i] = hi;
+      rope[2 * i + 1] = (float)(g - (double)hi);
+    }
+    e = ring.commit(wsp(ws.st_row0), st_bytes, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "upload static tables");
+    e = cudaMemsetAsync(wsp(ws.hdr), 0, 256, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(wsp(ws.counters), 0, 4 * (size_t)cfg.b * cfg.H, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+    device = dev;
+    cuda_ready = true;
+    return KVC_OK;
+  }
+
+  // Fill the decode state + prefix at the head of a dyn image.
+  void fill_state(unsigned char* img) {
+    kvc::DState* ds = reinterpret_cast<kvc::DState*>(img);
+    int64_t* P = reinterpret_cast<int64_t*>(img + ws.dyn_P);
+    decode_ok = true;
+    decode_err.clear();
+    P[0] = 0;
+    for (int s = 0; s < cfg.b; ++s) {
+      kvc::DecodeView v;
+      std::string err;
+      int64_t Lc = 0;
+      std::memset(&ds[s], 0, sizeof(kvc::DState));
+      if (bk.book.history(s) == 0) {
+        // no token yet: nothing to attend to, the sequence is skipped
+      } else if (bk.book.decode_view(s, v, err)) {
+        ds[s].len = (int32_t)v.len;
+        ds[s].begin = (int32_t)v.begin;
+        ds[s].mask_lo = (int32_t)v.mask_lo;
+        ds[s].mask_hi = (int32_t)v.mask_hi;
+        ds[s].qpos = v.qpos;
+        Lc = v.len - v.begin;
+      } else {
+        if (decode_ok) decode_err = err;
+        decode_ok = false;
+      }
+      P[s + 1] = P[s] + Lc;
+    }
+    R = (int64_t)cfg.H * P[cfg.b];
+  }
+};
+
+extern "C" {
+
+const char* kvc_status_string(kvc_status s) {
+  switch (s) {
+    case KVC_OK:
+      return "ok";
+    case KVC_ERR_INVALID_ARG:
+      return "invalid argument";
+    case KVC_ERR_UNSUPPORTED:
+      return "unsupported";
+    case KVC_ERR_CAPACITY:
+      return "capacity exceeded";
+    case KVC_ERR_SPAN:
+      return "span error";
+    case KVC_ERR_STATE:
+      return "state error";
+    case KVC_ERR_CUDA:
+      return "CUDA error";
+    case KVC_ERR_DEVICE_CHECK:
+      return "device check failed";
+    case KVC_ERR_TIMEOUT:
+      return "device wait timed out";
+    case KVC_ERR_NO_MEMORY:
+      return "out of host memory";
+  }
+  return "unknown status";
+}
+
+const char* kvc_last_error(void) { return g_last_error.c_str(); }
+
+// ------------------------------------------------------------------------------------------
+// book
+// ------------------------------------------------------------------------------------------
+
+kvc_status kvc_book_create(int b, kvc_policy policy, const int64_t* capacity, kvc_book** out) {
+  if (!out || !capacity || b <= 0) return fail(KVC_ERR_INVALID_ARG, "b must be positive, pointers non-NULL");
+  if (policy != KVC_POLICY_PAPER && policy != KVC_POLICY_KEEP_CL) return fail(KVC_ERR_INVALID_ARG, "policy");
+  for (int s = 0; s < b; ++s)
+    if (capacity[s] < 1) return fail(KVC_ERR_INVALID_ARG, "capacity[%d] < 1", s);
+  kvc_book* bk = new (std::nothrow) kvc_book(b, (kvc::Policy)policy, capacity);
+  if (!bk) return fail(KVC_ERR_NO_MEMORY, "book");
+  *out = bk;
+  return ok();
+}
+
+void kvc_book_destroy(kvc_book* book) { delete book; }
+
+static kvc_status book_check_append(const kvc::Book& B, const int32_t* n_new, const uint8_t* kinds) {
+  if (!n_new) return fail(KVC_ERR_INVALID_ARG, "n_new is NULL");
+  int64_t N = 0;
+  for (int s = 0; s < B.b(); ++s) N += n_new[s] > 0 ? n_new[s] : 0;
+  if (N > 0 && !kinds) return fail(KVC_ERR_INVALID_ARG, "kinds is NULL");
+  std::string err;
+  int code = 0;
+  if (!B.check_append(n_new, kinds, err, code)) return fail((kvc_status)code, "%s", err.c_str());
+  return KVC_OK;
+}
+
+kvc_status kvc_book_next_positions(const kvc_book* book, const int32_t* n_new, const uint8_t* kinds,
+                                   int32_t* pos_out) {
+  if (!book) return fail(KVC_ERR_INVALID_ARG, "book is NULL");
+  kvc_status st = book_check_append(book->book, n_new, kinds);
+  if (st != KVC_OK) return st;
+  if (!pos_out) return fail(KVC_ERR_INVALID_ARG, "pos_out is NULL");
+  book->book.next_positions(n_new, kinds, pos_out);
+  return ok();
+}
+
+kvc_status kvc_book_append(kvc_book* book, const int32_t* n_new, const uint8_t* kinds, const int32_t* pos) {
+  if (!book) return fail(KVC_ERR_INVALID_ARG, "book is NULL");
+  kvc_status st = book_check_append(book->book, n_new, kinds);
+  if (st != KVC_OK) return st;
+  if (!pos) return fail(KVC_ERR_INVALID_ARG, "pos is NULL");
+  book->book.apply_append(n_new, kinds, pos);
+  return ok();
+}
+
+kvc_status kvc_book_compress(kvc_book* book, const int32_t* seq, const int64_t* cl, const int64_t* cr, int n_spans) {
+  if (!book) return fail(KVC_ERR_INVALID_ARG, "book is NULL");
+  if (n_spans < 0 || (n_spans > 0 && (!seq || !cl || !cr))) return fail(KVC_ERR_INVALID_ARG, "span arrays");
+  std::vector<kvc::CompactSeq> plan;
+  std::string err;
+  if (!book->book.plan_compress(seq, cl, cr, n_spans, plan, err)) return fail(KVC_ERR_SPAN, "%s", err.c_str());
+  book->book.apply_compress(plan, seq, cl, n_spans);
+  return ok();
+}
+
+kvc_status kvc_book_pending_spans(const kvc_book* book, int seq, int64_t* cl, int64_t* cr, int64_t max, int64_t* n) {
+  if (!book || !n) return fail(KVC_ERR_INVALID_ARG, "NULL argument");
+  if (seq < 0 || seq >= book->book.b()) return fail(KVC_ERR_INVALID_ARG, "seq %d out of range", seq);
+  std::vector<std::pair<int64_t, int64_t>> v;
+  book->book.pending_spans(seq, v);
+  *n = (int64_t)v.size();
+  for (int64_t i = 0; i < std::min<int64_t>(max, (int64_t)v.size()); ++i) {
+    if (cl) cl[i] = v[i].first;
+    if (cr) cr[i] = v[i].second;
+  }
+  return ok();
+}
+
+kvc_status kvc_book_lengths(const kvc_book* book, int64_t* len_out, int64_t* attend_out) {
+  if (!book) return fail(KVC_ERR_INVALID_ARG, "book is NULL");
+  const kvc::Book& B = book->book;
+  for (int s = 0; s < B.b(); ++s) {
+    if (len_out) len_out[s] = B.stored(s);
+    if (attend_out) {
+      kvc::DecodeView v;
+      std::string err;
+      attend_out[s] = (B.history(s) > 0 && B.decode_view(s, v, err)) ? v.attended() : 0;
+    }
+  }
+  return ok();
+}
+
+kvc_status kvc_book_layout(const kvc_book* book, int seq, int64_t cap, uint8_t* kind_full, int32_t* pos_full,
+                           uint8_t* visible_full, int64_t* n_full, int32_t* stored_orig_idx, int32_t* stored_pos,
+                           int64_t* n_stored) {
+  if (!book || !n_full || !n_stored) return fail(KVC_ERR_INVALID_ARG, "NULL argument");
+  const kvc::Book& B = book->book;
+  if (seq < 0 || seq >= B.b()) return fail(KVC_ERR_INVALID_ARG, "seq %d out of range", seq);
+  const int64_t T = B.history(seq);
+  *n_full = T;
+  std::vector<int32_t> o, p;
+  B.stored_rows(seq, o, p);
+  *n_stored = (int64_t)o.size();
+  if (T > cap || (int64_t)o.size() > cap) return fail(KVC_ERR_CAPACITY, "cap %lld < %lld entries", (long long)cap, (long long)T);
+  if (kind_full) std::memcpy(kind_full, B.kinds(seq).data(), (size_t)T);
+  if (pos_full) std::memcpy(pos_full, B.positions(seq).data(), 4 * (size_t)T);
+  if (visible_full) B.visible(seq, visible_full);
+  if (stored_orig_idx) std::memcpy(stored_orig_idx, o.data(), 4 * o.size());
+  if (stored_pos) std::memcpy(stored_pos, p.data(), 4 * p.size());
+  return ok();
+}
+
+// ------------------------------------------------------------------------------------------
+// cache
+// ------------------------------------------------------------------------------------------
+
+kvc_status kvc_required_bytes(const kvc_config* cfg, size_t* k_bytes, size_t* v_bytes, size_t* meta_bytes_each,
+                              size_t* workspace_bytes) {
+  int64_t C = 0;
+  kvc_status st = check_config(cfg, &C);
+  if (st != KVC_OK) return st;
+  const size_t kv = (size_t)cfg->M * cfg->H * (size_t)C * cfg->d_head * 2;
+  if (k_bytes) *k_bytes = kv;
+  if (v_bytes) *v_bytes = kv;
+  if (meta_bytes_each) *meta_bytes_each = 4 * (size_t)C;
+  if (workspace_bytes) *workspace_bytes = ws_layout(cfg->b, cfg->H, cfg->d_head, cfg->rotary_dim, C).total;
+  return ok();
+}
+
+kvc_status kvc_create(const kvc_config* cfg, kvc_cache** out) {
+  if (!out) return fail(KVC_ERR_INVALID_ARG, "out is NULL");
+  int64_t C = 0;
+  kvc_status st = check_config(cfg, &C);
+  if (st != KVC_OK) return st;
+  if (!cfg->k_base || !cfg->v_base || !cfg->pos_base || !cfg->orig_base || !cfg->workspace)
+    return fail(KVC_ERR_INVALID_ARG, "device buffers must be non-NULL");
+  auto al = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 255u) == 0; };
+  if (!al(cfg->k_base) || !al(cfg->v_base) || !al(cfg->pos_base) || !al(cfg->orig_base) || !al(cfg->workspace))
+    return fail(KVC_ERR_INVALID_ARG, "device buffers must be 256-byte aligned");
+  const size_t need = ws_layout(cfg->b, cfg->H, cfg->d_head, cfg->rotary_dim, C).total;
+  if (cfg->workspace_bytes < need)
+    return fail(KVC_ERR_INVALID_ARG, "workspace_bytes=%zu < required %zu", cfg->workspace_bytes, need);
+  kvc_cache* c = new (std::nothrow) kvc_cache(*cfg, C);
+  if (!c) return fail(KVC_ERR_NO_MEMORY, "cache");
+  c->cfg.seq_capacity = c->cap.data();
+  *out = c;
+  return ok();
+}
+
+void kvc_destroy(kvc_cache* cache) { delete cache; }
+
+const kvc_book* kvc_get_book(const kvc_cache* cache) { return cache ? &cache->bk : nullptr; }
+
+kvc_status kvc_append(kvc_cache* c, int layer, const void* k, const void* v, const int32_t* n_new, const int32_t* pos,
+                      const uint8_t* kinds, void* stream_) {
+  if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  const int M = c->cfg.M;
+  if (layer < -1 || layer >= M) return fail(KVC_ERR_INVALID_ARG, "layer %d out of range [-1, %d)", layer, M);
+  if (!k || !v) return fail(KVC_ERR_INVALID_ARG, "k/v are NULL");
+  const bool starts = layer <= 0;
+  if (starts) {
+    if (c->layers_done != M)
+      return fail(KVC_ERR_STATE, "layers %d..%d of the previous tokens are not written yet", c->layers_done, M - 1);
+    kvc_status st = book_check_append(c->bk.book, n_new, kinds);
+    if (st != KVC_OK) return st;
+    int64_t N = 0;
+    for (int s = 0; s < c->cfg.b; ++s) N += n_new[s];
+    if (N > 0 && !pos) return fail(KVC_ERR_INVALID_ARG, "pos is NULL");
+  } else if (c->layers_done != layer) {
+    return fail(KVC_ERR_STATE, "layer %d appended out of order (expected %d)", layer, c->layers_done);
+  }
+  kvc_status st = c->ensure_cuda(stream);
+  if (st != KVC_OK) return st;
+  const kvc::Geometry g = c->geom();
+  if (starts) {
+    int64_t N = 0;
+    for (int s = 0; s < c->cfg.b; ++s) N += n_new[s];
+    // destination rows before the book moves on
+    std::vector<int64_t> row0(c->cfg.b), orig0(c->cfg.b);
+    for (int s = 0; s < c->cfg.b; ++s) {
+      row0[s] = c->bk.book.stored(s);
+      orig0[s] = c->bk.book.history(s);
+    }
+    const size_t bytes = c->ws.dyn_payload + sizeof(kvc::TokPlan) * (size_t)N;
+    cudaError_t e;
+    unsigned char* img = c->ring.reserve(bytes, &e);
+    if (!img) return cuda_fail(e, "staging");
+    c->bk.book.apply_append(n_new, kinds, pos);
+    c->fill_state(img);
+    kvc::TokPlan* tp = reinterpret_cast<kvc::TokPlan*>(img + c->ws.dyn_payload);
+    int64_t t = 0;
+    for (int s = 0; s < c->cfg.b; ++s) {
+      for (int i = 0; i < n_new[s]; ++i, ++t) {
+        tp[t].s = s;
+        tp[t].row = (int32_t)(row0[s] + i);
+        tp[t].pos = pos[t];
+        tp[t].orig = (int32_t)(orig0[s] + i);
+      }
+    }
+    e = c->ring.commit(c->wsp(c->ws.dyn), bytes, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "upload append plan");
+    c->batch_ntok = N;
+    c->layers_done = 0;
+  }
+  const int m0 = layer < 0 ? 0 : layer;
+  const int nl = layer < 0 ? M : 1;
+  if (c->batch_ntok > 0) {
+    const kvc::TokPlan* plan = reinterpret_cast<const kvc::TokPlan*>(c->wsp(c->ws.dyn + c->ws.dyn_payload));
+    cudaError_t e = kvc::launch_append(g, c->stat(), c->bufs(), plan, c->batch_ntok, m0, nl, m0 == 0, k, v, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "append kernel");
+    c->launches += 1;
+  }
+  c->layers_done = m0 + nl;
+  return ok();
+}
+
+kvc_status kvc_compress_spans(kvc_cache* c, const int32_t* seq, const int64_t* cl, const int64_t* cr, int n_spans,
+                              void* stream_) {
+  if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  if (n_spans < 0 || (n_spans > 0 && (!seq || !cl || !cr))) return fail(KVC_ERR_INVALID_ARG, "span arrays");
+  if (c->layers_done != c->cfg.M)
+    return fail(KVC_ERR_STATE, "layers %d..%d of the last tokens are not written yet", c->layers_done, c->cfg.M - 1);
+  std::vector<kvc::CompactSeq> plan;
+  std::string err;
+  if (!c->bk.book.plan_compress(seq, cl, cr, n_spans, plan, err)) return fail(KVC_ERR_SPAN, "%s", err.c_str());
+  if (n_spans == 0) return ok();
+  kvc_status st = c->ensure_cuda(stream);
+  if (st != KVC_OK) return st;
+  size_t n_ranges = 0;
+  int n_aff = 0;
+  for (auto& p : plan)
+    if (!p.drops.empty()) {
+      n_ranges += p.drops.size();
+      ++n_aff;
+    }
+  const size_t aff_bytes = sizeof(kvc::AffSeq) * (size_t)n_aff;
+  const size_t bytes = c->ws.dyn_payload + aff_bytes + 8 * n_ranges;
+  cudaError_t e;
+  unsigned char* img = c->ring.reserve(bytes, &e);
+  if (!img) return cuda_fail(e, "staging");
+  c->bk.book.apply_compress(plan, seq, cl, n_spans);
+  c->fill_state(img);
+  kvc::AffSeq* aff = reinterpret_cast<kvc::AffSeq*>(img + c->ws.dyn_payload);
+  int32_t* rg = reinterpret_cast<int32_t*>(img + c->ws.dyn_payload + aff_bytes);
+  int a = 0;
+  int32_t ro = 0;
+  for (auto& p : plan) {
+    if (p.drops.empty()) continue;
+    aff[a].s = p.s;
+    aff[a].len_old = (int32_t)p.len_old;
+    aff[a].len_new = (int32_t)p.len_new;
+    aff[a].first_row = (int32_t)p.first_row;
+    aff[a].range_off = ro;
+    aff[a].n_ranges = (int32_t)p.drops.size();
+    aff[a].pad0 = aff[a].pad1 = 0;
+    for (auto& d : p.drops) {
+      rg[2 * ro] = (int32_t)d.first;
+      rg[2 * ro + 1] = (int32_t)d.second;
+      ++ro;
+    }
+    ++a;
+  }
+  e = c->ring.commit(c->wsp(c->ws.dyn), bytes, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "upload compaction plan");
+  int launched = 0;
+  e = kvc::launch_compact(c->geom(), c->stat(), c->bufs(),
+                          reinterpret_cast<const kvc::AffSeq*>(c->wsp(c->ws.dyn + c->ws.dyn_payload)), n_aff,
+                          reinterpret_cast<const int32_t*>(c->wsp(c->ws.dyn + c->ws.dyn_payload + aff_bytes)),
+                          reinterpret_cast<int32_t*>(c->wsp(c->ws.dst_map)), stream, &launched);
+  c->launches += launched;
+  if (e != cudaSuccess) return cuda_fail(e, "compaction kernels");
+  return ok();
+}
+
+kvc_status kvc_decode_attention(kvc_cache* c, int layer, const void* q, float scale, float* out, void* stream_) {
+  if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  if (layer < 0 || layer >= c->cfg.M) return fail(KVC_ERR_INVALID_ARG, "layer %d out of range", layer);
+  if (!q || !out) return fail(KVC_ERR_INVALID_ARG, "q/out are NULL");
+  if (!std::isfinite(scale)) return fail(KVC_ERR_INVALID_ARG, "scale is not finite");
+  if (layer >= c->layers_done) return fail(KVC_ERR_STATE, "layer %d of the last tokens is not written yet", layer);
+  if (!c->cuda_ready) return fail(KVC_ERR_STATE, "nothing appended yet");
+  if (!c->decode_ok) return fail(KVC_ERR_STATE, "%s", c->decode_err.c_str());
+  if (c->R <= 0) return fail(KVC_ERR_STATE, "no sequence has a token to query");
+  kvc_status st = c->ensure_cuda(stream);
+  if (st != KVC_OK) return st;
+  kvc::DecodeArgs a;
+  a.layer = layer;
+  a.dstate = reinterpret_cast<const kvc::DState*>(c->wsp(c->ws.dyn));
+  a.P = reinterpret_cast<const int64_t*>(c->wsp(c->ws.dyn + c->ws.dyn_P));
+  a.R = c->R;
+  a.q = q;
+  a.out = out;
+  a.scale = scale;
+  a.partials = reinterpret_cast<float*>(c->wsp(c->ws.partials));
+  a.counters = reinterpret_cast<int*>(c->wsp(c->ws.counters));
+  a.wait_limit_ns = 2000000000ull;
+  int grid = 0;
+  cudaError_t e = kvc::launch_decode(c->geom(), c->stat(), c->bufs(), a, c->num_sms, stream, &grid);
+  if (e != cudaSuccess) return cuda_fail(e, "decode kernel");
+  c->launches += grid > 0 ? 1 : 0;
+  return ok();
+}
+
+kvc_status kvc_masked_reference_layout(kvc_cache* c, int seq, int64_t cap, uint8_t* kind_full, int32_t* pos_full,
+                                       uint8_t* visible_full, int64_t* n_full, int32_t* stored_orig_idx,
+                                       int32_t* stored_pos, int64_t* n_stored, void* stream_) {
+  if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  int64_t ns = 0;
+  kvc_status st = kvc_book_layout(&c->bk, seq, cap, kind_full, pos_full, visible_full, n_full, nullptr, nullptr, &ns);
+  if (st != KVC_OK) return st;
+  *n_stored = ns;
+  if (ns == 0) return ok();
+  st = c->ensure_cuda(stream);
+  if (st != KVC_OK) return st;
+  cudaError_t e = cudaSuccess;
+  if (stored_orig_idx)
+    e = cudaMemcpyAsync(stored_orig_idx, c->cfg.orig_base + c->off[seq], 4 * (size_t)ns, cudaMemcpyDeviceToHost,
+                        stream);
+  if (e == cudaSuccess && stored_pos)
+    e = cudaMemcpyAsync(stored_pos, c->cfg.pos_base + c->off[seq], 4 * (size_t)ns, cudaMemcpyDeviceToHost, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "read back stored rows");
+  return ok();
+}
+
+kvc_status kvc_device_status(kvc_cache* c, void* stream_, int32_t* word) {
+  if (!c || !word) return fail(KVC_ERR_INVALID_ARG, "NULL argument");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  *word = 0;
+  if (!c->cuda_ready) return ok();
+  int32_t w = 0;
+  cudaError_t e = cudaMemcpyAsync(&w, c->wsp(c->ws.hdr), 4, cudaMemcpyDeviceToHost, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "read status");
+  *word = w;
+  if (w == 0) return ok();
+  e = cudaMemsetAsync(c->wsp(c->ws.hdr), 0, 4, stream);
+  // a timed-out decode may leave split-K arrival counters behind: start them from zero again
+  if (e == cudaSuccess && (w & kvc::STATUS_TIMEOUT))
+    e = cudaMemsetAsync(c->wsp(c->ws.counters), 0, 4 * (size_t)c->cfg.b * c->cfg.H, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "clear status");
+  if (w & kvc::STATUS_TIMEOUT) return fail(KVC_ERR_TIMEOUT, "a kernel's bounded wait ran out (status 0x%x)", w);
+  return fail(KVC_ERR_DEVICE_CHECK, "a kernel's consistency check failed (status 0x%x)", w);
+}
+
+int64_t kvc_launch_count(const kvc_cache* c) { return c ? c->launches : 0; }
+
+}  // extern "C"

@@ -1,0 +1,245 @@
+"""The C ABI on the host (CPU only): exported symbols, argument/state errors, and the span book
+(a2: span bookkeeping, positions, stored rows, mask) against the fp64 oracle, bit-exact."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle as orc
+import paper_2310_08152_gb300 as kvc
+from paper_2310_08152_gb300 import _lib
+from synth import workloads as wl
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+NORMAL, CL, CR = kvc.NORMAL, kvc.CL, kvc.CR
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "kvc.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(kvc_[a-z_]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_function():
+    names = declared_functions()
+    assert len(names) >= 20
+    L = kvc.lib()
+    for n in names:
+        assert hasattr(L, n), n
+    assert sorted(n for n, _, _ in _lib.SIGNATURES) == names
+
+
+def test_status_strings():
+    L = kvc.lib()
+    for s in range(10):
+        assert L.kvc_status_string(s)
+    assert L.kvc_status_string(0) == b"ok"
+
+
+# --------------------------------------------------------------------------------------------
+# book vs oracle
+# --------------------------------------------------------------------------------------------
+
+def _random_kinds(rng, n, open_=False):
+    kinds = np.zeros(n, np.uint8)
+    for t in range(n):
+        r = rng.random()
+        if not open_ and r < 0.12:
+            kinds[t] = CL
+            open_ = True
+        elif open_ and r < 0.15:
+            kinds[t] = CR
+            open_ = False
+    return kinds, open_
+
+
+@pytest.mark.parametrize("policy", [kvc.POLICY_PAPER, kvc.POLICY_KEEP_CL])
+def test_book_matches_oracle_random_histories(policy):
+    rng = np.random.default_rng(20)
+    b = 4
+    cap = np.full(b, 4000, np.int64)
+    book = kvc.Book(b, cap, policy)
+    hist = [np.zeros(0, np.uint8) for _ in range(b)]
+    freed = [[] for _ in range(b)]
+    open_ = [False] * b
+    for rnd in range(40):
+        n_new = rng.integers(0, 12, size=b).astype(np.int32)
+        parts = []
+        for s in range(b):
+            k, open_[s] = _random_kinds(rng, int(n_new[s]), open_[s])
+            parts.append(k)
+        kinds = np.concatenate(parts)
+        pos = book.append(n_new, kinds)
+        # positions continue each history with the tie rule
+        off = 0
+        for s in range(b):
+            hist[s] = np.concatenate([hist[s], parts[s]])
+            expect = orc.tied_positions(hist[s])[hist[s].size - n_new[s]:]
+            assert np.array_equal(pos[off:off + n_new[s]], expect)
+            off += n_new[s]
+        # free a random subset of the pending spans
+        seq, cl, cr = [], [], []
+        for s in range(b):
+            for a, c in book.pending_spans(s):
+                if rng.random() < 0.6:
+                    seq.append(s)
+                    cl.append(a)
+                    cr.append(c)
+                    freed[s].append((a, c))
+        if seq:
+            book.compress(seq, cl, cr)
+        ln, at = book.lengths()
+        for s in range(b):
+            lay = book.layout(s)
+            T = hist[s].size
+            assert np.array_equal(lay["kinds"], hist[s])
+            rows = orc.stored_rows(T, freed[s], policy)
+            assert np.array_equal(lay["stored_orig"], rows)
+            assert ln[s] == rows.size
+            assert np.array_equal(lay["stored_pos"], orc.tied_positions(hist[s])[rows])
+            closed, _ = orc.pair_spans(hist[s])
+            assert book.pending_spans(s) == [sp for sp in closed if sp not in freed[s]]
+            if T:
+                vis = orc.visible(hist[s], T - 1, policy)
+                assert np.array_equal(lay["visible"], vis)
+                # rows the next decode reads: the visible ones, when every hidden row sits in one run
+                hidden = set(rows.tolist()) - set(np.nonzero(vis)[0].tolist())
+                idx = sorted(np.searchsorted(rows, list(hidden)))
+                one_run = not idx or idx[-1] - idx[0] + 1 == len(idx)
+                if one_run or hist[s][T - 1] == CL:
+                    # the decode reads exactly the stored rows the mask shows (a <CR> query whose span
+                    # was already freed sees the rows that are left)
+                    assert at[s] == vis[rows].sum()
+                else:
+                    assert at[s] == 0
+
+
+def test_book_workload_counts():
+    for w in (wl.tiny(), wl.opt13b(b=2), wl.rope3b(45, b=1)):
+        book = kvc.Book(w.b, w.capacity(0), kvc.POLICY_PAPER)
+        book.append(w.prompt_len.astype(np.int32), np.concatenate(w.prompt_kinds))
+        seq = [s for s in range(w.b) for _ in w.prompt_spans[s]]
+        cl = [a for s in range(w.b) for a, _ in w.prompt_spans[s]]
+        cr = [c for s in range(w.b) for _, c in w.prompt_spans[s]]
+        book.compress(seq, cl, cr)
+        ln, at = book.lengths()
+        L = int(w.prompt_len[0])
+        I = w.prompt_spans[0][0][1] - w.prompt_spans[0][0][0] - 1
+        assert np.all(ln == (L // 64) * (64 - I - 1))
+
+
+# --------------------------------------------------------------------------------------------
+# host-side errors
+# --------------------------------------------------------------------------------------------
+
+def _err(fn, *a):
+    with pytest.raises(kvc.KvcError) as e:
+        fn(*a)
+    return e.value.status
+
+
+def test_book_span_errors_leave_state_unchanged():
+    book = kvc.Book(2, [100, 100])
+    book.append([3, 1], [NORMAL, CL, NORMAL, NORMAL])
+    before = (book.layout(0), book.layout(1), book.lengths())
+    assert _err(book.append, [1, 0], [CL]) == 4          # <CL> inside the open span of sequence 0
+    assert _err(book.append, [0, 1], [CR]) == 4          # <CR> without an open span in sequence 1
+    assert _err(book.append, [0, 200], [NORMAL] * 200) == 3  # capacity
+    assert _err(book.append, [1, 0], [7]) == 1           # not a kind
+    assert _err(book.append, [-1, 0], []) == 1
+    after = (book.layout(0), book.layout(1), book.lengths())
+    for x, y in zip(before[:2], after[:2]):
+        for key in x:
+            assert np.array_equal(x[key], y[key])
+    book.append([2, 0], [NORMAL, CR])
+    assert book.pending_spans(0) == [(1, 4)]
+    assert _err(book.compress, [0], [0], [4]) == 4       # not a span
+    assert _err(book.compress, [0], [1], [3]) == 4       # wrong <CR>
+    assert _err(book.compress, [0, 0], [1, 1], [4, 4]) == 4  # listed twice
+    assert _err(book.compress, [5], [1], [4]) == 4       # sequence out of range
+    book.compress([0], [1], [4])
+    assert _err(book.compress, [0], [1], [4]) == 4       # already freed
+    assert book.lengths()[0][0] == 2
+
+
+def test_book_open_span_cannot_be_freed():
+    book = kvc.Book(1, [50])
+    book.append([3], [NORMAL, CL, NORMAL])
+    assert _err(book.compress, [0], [1], [3]) == 4
+
+
+def test_decode_view_needs_spans_freed():
+    # two closed spans that are not freed leave two hidden runs: the next decode must refuse
+    book = kvc.Book(1, [50])
+    book.append([9], [NORMAL, CL, NORMAL, CR, NORMAL, CL, NORMAL, CR, NORMAL])
+    ln, at = book.lengths()
+    assert at[0] == 0
+    book.compress([0], [1], [3])
+    ln, at = book.lengths()
+    assert at[0] == orc.visible(np.array([0, 1, 0, 2, 0, 1, 0, 2, 0], np.uint8), 8).sum()
+
+
+def test_cache_config_errors_on_host():
+    cfg, cap = kvc.make_config(2, 4, 72, [16, 16])
+    assert _err(kvc.kvc_required_bytes, cfg) == 2        # d_head not built
+    cfg, cap = kvc.make_config(2, 4, 64, [16, 16], rotary_dim=24)
+    assert _err(kvc.kvc_required_bytes, cfg) == 2        # rotary_dim not a multiple of 16
+    cfg, cap = kvc.make_config(2, 4, 64, [16, 0])
+    assert _err(kvc.kvc_required_bytes, cfg) == 1
+    cfg, cap = kvc.make_config(2, 4, 64, [16, 16])
+    sizes = kvc.kvc_required_bytes(cfg)
+    assert sizes["k"] == 2 * 4 * 32 * 64 * 2 and sizes["meta"] == 32 * 4
+    assert _err(kvc.kvc_create, cfg) == 1                # NULL device buffers
+    cfg.k_base = cfg.v_base = cfg.pos_base = cfg.orig_base = cfg.workspace = 0x1000 + 8
+    cfg.workspace_bytes = sizes["workspace"]
+    assert _err(kvc.kvc_create, cfg) == 1                # unaligned
+
+
+def test_cache_validates_before_any_device_work():
+    # Fake (never dereferenced) addresses: every call below must fail on the host before touching CUDA.
+    cfg, cap = kvc.make_config(2, 4, 64, [16, 16])
+    sizes = kvc.kvc_required_bytes(cfg)
+    cfg.k_base = cfg.v_base = cfg.pos_base = cfg.orig_base = cfg.workspace = 1 << 40
+    cfg.workspace_bytes = sizes["workspace"]
+    h = kvc.kvc_create(cfg)
+    try:
+        fake = 1 << 40
+        L = kvc.lib()
+        n_new = np.array([1, 1], np.int32)
+        pos = np.zeros(2, np.int32)
+        assert L.kvc_append(h, 5, fake, fake, n_new.ctypes.data, pos.ctypes.data, np.uint8([0, 0]).ctypes.data,
+                            None) == 1
+        assert L.kvc_append(h, -1, fake, fake, n_new.ctypes.data, pos.ctypes.data, np.uint8([2, 0]).ctypes.data,
+                            None) == 4
+        big = np.array([17, 0], np.int32)
+        assert L.kvc_append(h, -1, fake, fake, big.ctypes.data, np.zeros(17, np.int32).ctypes.data,
+                            np.zeros(17, np.uint8).ctypes.data, None) == 3
+        assert L.kvc_append(h, 1, fake, fake, None, None, None, None) == 5   # layer 1 before layer 0
+        assert L.kvc_decode_attention(h, 0, fake, ctypes.c_float(0.125), fake, None) == 5  # nothing appended
+        assert L.kvc_decode_attention(h, 9, fake, ctypes.c_float(0.125), fake, None) == 1
+        assert L.kvc_compress_spans(h, np.int32([0]).ctypes.data, np.int64([0]).ctypes.data,
+                                    np.int64([1]).ctypes.data, 1, None) == 4
+        assert b"span" in L.kvc_last_error() or b"closed" in L.kvc_last_error()
+    finally:
+        kvc.kvc_destroy(h)
+
+
+def test_cache_fails_loudly_without_a_gpu():
+    import torch
+
+    if torch.cuda.is_available():
+        pytest.skip("only meaningful where no GPU exists (it would dereference fake addresses)")
+    cfg, cap = kvc.make_config(1, 2, 64, [8])
+    sizes = kvc.kvc_required_bytes(cfg)
+    cfg.k_base = cfg.v_base = cfg.pos_base = cfg.orig_base = cfg.workspace = 1 << 40
+    cfg.workspace_bytes = sizes["workspace"]
+    h = kvc.kvc_create(cfg)
+    try:
+        L = kvc.lib()
+        rc = L.kvc_append(h, -1, 1 << 40, 1 << 40, np.int32([1]).ctypes.data, np.int32([0]).ctypes.data,
+                          np.uint8([0]).ctypes.data, None)
+        assert rc == 6  # KVC_ERR_CUDA: no silent CPU path
+    finally:
+        kvc.kvc_destroy(h)

@@ -1,0 +1,60 @@
+"""Parity at the workloads' full sizes, in the launch configuration the benchmark times: compaction
+metadata of every sequence bit-exact, sampled cache rows bit-exact, and sampled decode outputs
+(layers first/middle/last, sequences first/middle/last, every head) within tolerance of the fp64
+oracle at the first step, right after compactions and at the last step checked."""
+import numpy as np
+import pytest
+import torch
+
+import harness
+import oracle.workload as ow
+from synth import workloads as wl
+
+from _parity import check_metadata, check_rows, compare
+
+pytestmark = pytest.mark.gpu
+
+
+def _full(w, steps, check_at, rope=False):
+    run = harness.Runner(w, steps)
+    run.load_prompt()
+    check_metadata(run, 0)
+    seqs = sorted({0, w.b // 2, w.b - 1})
+    layers = sorted({0, w.M // 2, w.M - 1})
+    for s in seqs:
+        check_rows(run, 0, layers[-1], s, [0, w.H - 1], check_k=not rope)
+    out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device=run.device)
+    for g in range(steps):
+        inp = run.make_step_inputs(g)
+        closed = run.step(inp, out)
+        if g in check_at:
+            torch.cuda.synchronize()
+            o = out.cpu().numpy()
+            for m in layers:
+                ref = ow.expected_decode(w, g + 1, m, seqs)
+                compare(o[m][seqs], ref, f"{w.name} step {g} layer {m}")
+        if closed:
+            check_metadata(run, g + 1)
+    assert run.cache.device_status() == 0
+    return run
+
+
+def test_full_opt13b_shaped():
+    # 128 steps as in the workload: compactions after g = 32, 65, 98
+    _full(wl.opt13b(), 128, check_at={0, 1, 32, 33, 34, 66, 127})
+
+
+def test_full_opt27b_shaped():
+    _full(wl.opt27b(), 64, check_at={0, 7, 8, 52, 53, 63})
+
+
+@pytest.mark.parametrize("interior", [19, 32, 45])
+def test_full_rope3b_shaped(interior):
+    _full(wl.rope3b(interior), 8, check_at={0, 7}, rope=True)
+
+
+def test_full_ragged():
+    w = wl.ragged()
+    run = _full(w, 32, check_at={0, 15, 31})
+    ln = run.cache.lengths()[0]
+    assert ln.max() > 4000 and ln.min() < 300

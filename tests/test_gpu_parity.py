@@ -1,0 +1,200 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle, at sizes the oracle finishes in
+seconds: several tiles per segment, split segments, ragged tails, every step kind (normal, <CL>
+query, open-span queries, <CR> query, compaction right after it), both policies, every built d_head."""
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+import harness
+import oracle as orc
+import oracle.workload as ow
+import paper_2310_08152_gb300 as kvc
+import synth
+from synth import workloads as wl
+
+from _parity import MAX_ABS, check_metadata, check_rows, compare, run_workload
+
+pytestmark = pytest.mark.gpu
+
+
+def test_device_generator_matches_host():
+    rng = np.random.default_rng(1)
+    for dtype, sigma in (("f16", 1.0), ("bf16", 80 ** -0.5)):
+        t = rng.integers(0, 9000, size=300).astype(np.int32)
+        s = rng.integers(0, 128, size=300).astype(np.int32)
+        sc = synth.scale_for(sigma)
+        tag = synth.tag(synth.V_TENSOR, 17)
+        host = synth.fill_tokens_host(77, dtype, sc, tag, t, s, 5, 80)
+        out = torch.empty(300 * 5 * 80, dtype=torch.int16, device="cuda")
+        synth.fill_tokens_cuda(77, dtype, sc, tag, torch.from_numpy(t).cuda(), torch.from_numpy(s).cuda(), 5, 80, out)
+        assert np.array_equal(out.cpu().numpy().view(np.uint16).reshape(300, 5, 80), host)
+
+
+def test_tiny_config_every_output():
+    run, worst = run_workload(wl.tiny(), steps=1)
+    for s in range(2):
+        check_rows(run, 1, 0, s, range(4))
+    assert worst[0] <= MAX_ABS
+
+
+def test_opt13b_shaped_small():
+    # H=32, d=64, fp16: <CL> query at g=0 and 33, open-span queries, <CR> at g=32 then compaction
+    w = wl.opt13b(b=3, L=640, M=2)
+    run, _ = run_workload(w, steps=36)
+    for s in range(3):
+        check_rows(run, 36, 1, s, [0, 31])
+
+
+def test_opt27b_shaped_small():
+    # d=80, bf16, q std d^-1/2 with scale 1; span opened at g=7, closed at g=52
+    w = wl.opt27b(b=3, L=704, M=2)
+    run, _ = run_workload(w, steps=54, check_steps={0, 7, 8, 30, 51, 52, 53})
+    check_rows(run, 54, 0, 2, [5])
+
+
+@pytest.mark.parametrize("interior", [19, 32, 45])
+def test_rope3b_shaped_small(interior):
+    w = wl.rope3b(interior, b=3, L=640, M=2)
+    run, _ = run_workload(w, steps=6)
+    check_rows(run, 6, 1, 0, [3], check_k=False)  # K is stored rotated
+
+
+def test_ragged_small():
+    w = wl.ragged(b=6, lmin=64, lmax=900, M=2, steps=32)
+    run_workload(w, steps=32, check_steps={0, 10, 20, 31})
+
+
+def test_keep_cl_policy():
+    w = wl.opt13b(b=2, L=384, M=1)
+    run_workload(w, steps=35, policy=orc.POLICY_KEEP_CL)
+
+
+@pytest.mark.parametrize("d,dtype", [(96, "f16"), (128, "bf16"), (64, "bf16"), (80, "f16")])
+def test_every_built_head_dim(d, dtype):
+    w = dataclasses.replace(wl.opt13b(b=2, L=448, M=2), d=d, dtype=dtype, name=f"d{d}-{dtype}")
+    run_workload(w, steps=34, check_steps={0, 1, 31, 32, 33})
+
+
+def test_rope_partial_rotary_dim():
+    w = dataclasses.replace(wl.rope3b(32, b=2, L=384, M=1), rotary_dim=32, name="rope-partial")
+    run_workload(w, steps=3)
+
+
+def test_long_segments_split_over_many_ctas():
+    # one long sequence and a short one: stream-K splits the long segments across many CTAs
+    w = dataclasses.replace(wl.opt13b(b=2, L=64, M=1), name="long")
+    kinds_long, spans_long = wl.block_kinds(9000, 32)
+    kinds_short, spans_short = wl.block_kinds(70, 8)
+    w.prompt_kinds = [kinds_long, kinds_short]
+    w.prompt_spans = [spans_long, spans_short]
+    run_workload(w, steps=2)
+
+
+def test_sequences_without_tokens_are_skipped():
+    w = wl.opt13b(b=3, L=320, M=1)
+    run = harness.Runner(w, steps=1)
+    n_new = np.array([320, 0, 320], np.int32)
+    kinds = np.concatenate([w.prompt_kinds[0], w.prompt_kinds[2]])
+    N = 640
+    k = torch.empty(N * w.H * w.d, dtype=torch.float16, device="cuda")
+    v = torch.empty_like(k)
+    tok_t = torch.from_numpy(np.concatenate([np.arange(320), np.arange(320)]).astype(np.int32)).cuda()
+    tok_s = torch.from_numpy(np.repeat(np.int32([0, 2]), 320)).cuda()
+    run._fill(synth.K_TENSOR, 0, tok_t, tok_s, k, run.kv_scale)
+    run._fill(synth.V_TENSOR, 0, tok_t, tok_s, v, run.kv_scale)
+    run.cache.append(k, v, n_new, kinds)
+    q = torch.empty(1, 3, w.H, w.d, dtype=torch.float16, device="cuda")
+    run._fill(synth.Q_TENSOR, 0, torch.full((3,), 319, dtype=torch.int32, device="cuda"),
+              torch.arange(3, dtype=torch.int32, device="cuda"), q[0], run.q_scale)
+    out = torch.full((3, w.H, w.d), float("nan"), device="cuda")
+    # two pending spans hide more than one run: the decode must refuse until they are freed
+    with pytest.raises(kvc.KvcError) as e:
+        run.cache.decode_attention(0, q[0], w.scale, out)
+    assert e.value.status == 5
+    run.cache.compress_spans([s for s in (0, 2) for _ in w.prompt_spans[s]],
+                             [a for s in (0, 2) for a, _ in w.prompt_spans[s]],
+                             [c for s in (0, 2) for _, c in w.prompt_spans[s]])
+    run.cache.decode_attention(0, q[0], w.scale, out)
+    torch.cuda.synchronize()
+    o = out.cpu().numpy()
+    assert np.isnan(o[1]).all()  # untouched
+    kinds0, pos0 = w.prompt_kinds[0], orc.tied_positions(w.prompt_kinds[0])
+    K, V = ow.kv_bits(w, 0, 0, 320)
+    ref = orc.masked_decode([kinds0], [pos0], [K], [V], ow.q_bits(w, 0, 0, 319)[None], "f16", w.scale)
+    compare(o[0:1], ref)
+    assert run.cache.device_status() == 0
+
+
+def test_capacity_edge_and_errors_through_the_cache():
+    w = dataclasses.replace(wl.opt13b(b=1, L=128, M=1), name="no-spans")
+    w.prompt_kinds = [np.zeros(128, np.uint8)]
+    w.prompt_spans = [[]]
+    run = harness.Runner(w, steps=2)
+    run.load_prompt()
+    out = torch.empty(1, 1, w.H, w.d, device="cuda")
+    for g in range(2):
+        run.step(run.make_step_inputs(g), out)
+    # the cache is full now (capacity = L + 2): one more row must be refused on the host
+    inp = run.make_step_inputs(2)
+    with pytest.raises(kvc.KvcError) as e:
+        run.cache.append(inp.kv_k, inp.kv_v, np.ones(1, np.int32), np.zeros(1, np.uint8))
+    assert e.value.status == 3
+    # compaction of something that is not a closed span
+    with pytest.raises(kvc.KvcError) as e:
+        run.cache.compress_spans([0], [7], [40])
+    assert e.value.status == 4
+    assert run.cache.device_status() == 0
+
+
+def test_span_at_history_start_and_empty_interior():
+    # <CL> at index 0 (first dropped row is row 0) and, under KEEP_CL, a <CL><CR> pair with nothing inside
+    w = dataclasses.replace(wl.opt13b(b=2, L=64, M=1), name="edges")
+    k0 = np.zeros(200, np.uint8)
+    k0[0], k0[9] = wl.CL, wl.CR
+    k0[50], k0[51] = wl.CL, wl.CR
+    k1 = np.zeros(150, np.uint8)
+    k1[149 - 5], k1[149] = wl.CL, wl.CR
+    w.prompt_kinds = [k0, k1]
+    w.prompt_spans = [[(0, 9), (50, 51)], [(144, 149)]]
+    for policy in (orc.POLICY_PAPER, orc.POLICY_KEEP_CL):
+        run_workload(w, steps=2, policy=policy)
+
+
+def test_per_layer_append_equals_all_layer_append():
+    w = wl.opt13b(b=2, L=192, M=3)
+    a = harness.Runner(w, steps=1)
+    a.load_prompt()  # per-layer appends
+    b = harness.Runner(w, steps=1)
+    # all layers in one call
+    n_new = b.L.astype(np.int32)
+    N = int(n_new.sum())
+    tok_t = torch.from_numpy(np.concatenate([np.arange(L, dtype=np.int32) for L in b.L])).cuda()
+    tok_s = torch.from_numpy(np.repeat(np.arange(w.b, dtype=np.int32), b.L)).cuda()
+    k = torch.empty(w.M, N * w.H * w.d, dtype=torch.float16, device="cuda")
+    v = torch.empty_like(k)
+    for m in range(w.M):
+        b._fill(synth.K_TENSOR, m, tok_t, tok_s, k[m], b.kv_scale)
+        b._fill(synth.V_TENSOR, m, tok_t, tok_s, v[m], b.kv_scale)
+    b.cache.append(k, v, n_new, np.concatenate(w.prompt_kinds))
+    b.compress_prompt()
+    torch.cuda.synchronize()
+    for s in range(w.b):
+        la, lb = a.cache.masked_reference_layout(s), b.cache.masked_reference_layout(s)
+        n = la["stored_orig"].size
+        assert np.array_equal(la["stored_orig"], lb["stored_orig"])
+        for m in range(w.M):
+            for h in (0, 17, 31):
+                for pa, pb in ((a.cache.k_plane(m), b.cache.k_plane(m)), (a.cache.v_plane(m), b.cache.v_plane(m))):
+                    assert torch.equal(a.cache.stream_rows(pa, s, h, n), b.cache.stream_rows(pb, s, h, n))
+
+
+def test_launch_counter_counts_kernels():
+    w = wl.tiny()
+    run = harness.Runner(w, steps=1)
+    run.load_prompt()  # one append (M=1) + scan + move
+    assert run.cache.launch_count == 3
+    out = torch.empty(1, 2, 4, 64, device="cuda")
+    run.step(run.make_step_inputs(0), out)  # append + decode
+    assert run.cache.launch_count == 5
