@@ -43,6 +43,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="budget of the CPU-baseline sample")
+    ap.add_argument("--layers", type=int, default=0, help="override the layer count (small profiling runs)")
     return ap.parse_args()
 
 
@@ -389,6 +390,10 @@ def main():
     from synth import workloads as wl
 
     w = wl.by_name(args.workload)
+    if args.layers:
+        import dataclasses
+
+        w = dataclasses.replace(w, M=args.layers, name=f"{w.name}-M{args.layers}")
     if args.impl == "reference":
         run_reference(args, w)
     else:
