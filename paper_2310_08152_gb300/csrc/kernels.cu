@@ -5,11 +5,12 @@
 //                         in-place move of the position / history-index metadata
 //   compact_move_kernel   in-place, ascending, 16-byte vectorised row moves of every
 //                         (layer, K/V, head) stream of the affected sequences
-//   decode_kernel         split-K single-query attention over the kept rows: a producer warp streams
-//                         K/V tiles into shared memory with 1-D TMA bulk copies (cp.async.bulk +
-//                         mbarrier), eight consumer warps do fp32 dot products, warp-shuffle
-//                         reductions and an online softmax; pieces of a split row range are merged
-//                         by a log-sum-exp combine done by the last CTA to finish (arrival counter).
+//   decode_kernel         split-K single-query attention over the kept rows: every warp is a worker
+//                         that streams its share of the rows through a ring of shared-memory
+//                         stages with 1-D TMA bulk copies (cp.async.bulk + mbarrier), does packed
+//                         fp32 dot products, warp-shuffle reductions and an online softmax; the
+//                         parts of a split (sequence, head) are merged by a log-sum-exp combine done
+//                         by the last worker to finish (arrival counter).
 //
 // No tensor cores: one query per (sequence, head) makes decode a GEMV (1 flop per byte read), far
 // below any tensor-core ridge; the kernels are bound by HBM bandwidth.
@@ -61,7 +62,7 @@ __device__ __forceinline__ void rope_sincos(int32_t pos, float2 g, float* s, flo
 }
 
 // ---------------------------------------------------------------------------------------------
-// PTX helpers: mbarrier, 1-D bulk copy (TMA), named barrier, global timer
+// PTX helpers: mbarrier, 1-D bulk copy (TMA), global timer
 // ---------------------------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -73,9 +74,6 @@ __device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
                : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
@@ -107,9 +105,6 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
                    smem_addr(dst)),
                "l"(src), "r"(bytes), "r"(smem_addr(bar))
                : "memory");
-}
-__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -330,35 +325,43 @@ __global__ void __launch_bounds__(kMoveThreads) compact_move_kernel(Geometry g, 
 // ---------------------------------------------------------------------------------------------
 // a5 + a6: decode
 // ---------------------------------------------------------------------------------------------
-// Lane geometry: LPR lanes share one row; lane t reads NV vectors of VB bytes at vector indices
-// t + LPR*i.  Chosen so that the lanes of one shared-memory wavefront (8 lanes for 16-byte, 16
-// lanes for 8-byte accesses) hit distinct banks for the row size at hand.
+// Work split ("stream-K" over rows): the attended rows of every (sequence, head) segment are
+// concatenated and cut into NW equal contiguous ranges, one per warp.  A warp is an independent
+// flash-decoding worker: it streams its rows through its own ring of shared-memory stages (1-D TMA
+// bulk copies issued by its lane 0, completion on an mbarrier), keeps an online softmax, and at
+// the end of each piece (its part of one segment) either writes the output row (the whole segment
+// was its own) or a partial (m, l, o); the last of a segment's workers to finish combines them.
+//
+// Lane geometry: LPR lanes share one row, lane t of a row holds NV 16-byte chunks.  Row group g
+// (lane / LPR) reads chunk t*NV + (i + A*g + B*t) mod NV at step i: the rotation makes every
+// 8-lane shared-memory wavefront hit 8 distinct bank groups; q is staged per lane in the same
+// rotated order, and partial outputs are written back to their natural columns through shared
+// memory, so the rotation never needs register indexing.
 template <int D>
 struct Lanes {
-  static constexpr int RB = D * 2;
-  static constexpr int MODE = (RB % 128 == 0) ? 0 : ((RB % 128 == 64) ? 1 : 2);
-  static constexpr int VB = MODE == 0 ? 16 : 8;
-  static constexpr int LPR = MODE == 2 ? 4 : 8;
-  static constexpr int NV = RB / (VB * LPR);
-  static constexpr int EPV = VB / 2;
-  static constexpr int EPL = NV * EPV;
-  static constexpr int RPI = 32 / LPR;
-  static_assert(RB % 32 == 0, "d_head must be a multiple of 16");
-  static_assert(NV * VB * LPR == RB, "row must split evenly over the lanes");
+  static constexpr int RB = D * 2;                        // row bytes
+  static constexpr int CH = D / 8;                        // 16-byte chunks per row
+  static constexpr int LPR = (D == 96 || D == 128) ? 4 : 2;
+  static constexpr int NV = CH / LPR;                     // chunks per lane
+  static constexpr int EPL = NV * 8;                      // elements per lane
+  static constexpr int RPI = 32 / LPR;                    // rows per warp step
+  static constexpr int A = (D == 64 || D == 128) ? 1 : 0;
+  static constexpr int B = (D == 128) ? 1 : 0;
+  static_assert(D % 16 == 0 && CH % LPR == 0, "unsupported d_head");
 };
 
 template <int D>
 struct DecodeCfg {
   using L = Lanes<D>;
-  static constexpr int NCW = 8;   // consumer warps
-  static constexpr int TR = 64;   // rows per tile
-  static constexpr int TILE = TR * L::RB;
-  static constexpr int S = (100 * 1024) / (2 * TILE);  // pipeline stages
-  static constexpr int KPT = TR / (NCW * L::RPI);       // rows per lane per tile
-  static constexpr int THREADS = (NCW + 1) * 32;
-  static constexpr int SMEM = 2 * S * TILE + 2 * S * 8 + 2 * NCW * D * 4 + 2 * NCW * 2 * 4;
-  static_assert(KPT >= 1 && KPT * NCW * L::RPI == TR, "tile must split evenly over the warps");
-  static_assert(S >= 2, "need at least two stages");
+  static constexpr int KPT = 2;                 // rows per lane per tile
+  static constexpr int TR = KPT * L::RPI;       // rows per tile
+  static constexpr int TILE = TR * L::RB;       // bytes per K (or V) tile
+  static constexpr int S = 3;                   // stages per warp
+  static constexpr int WARPS = 4;               // warps per CTA
+  static constexpr int THREADS = WARPS * 32;
+  static constexpr int WARP_SMEM = (2 * S * TILE + D * 4 + S * 8 + 127) / 128 * 128;
+  static constexpr int SMEM = WARPS * WARP_SMEM;
+  static_assert(L::RPI * D * 4 <= TILE, "reduction scratch must fit in one tile");
 };
 
 struct DecodeDev {
@@ -367,7 +370,7 @@ struct DecodeDev {
   const DState* ds;
   const int64_t* P;
   int64_t R;
-  int G;
+  int NW;  // workers (warps)
   const uint16_t* q;
   float* out;
   float* partials;
@@ -377,42 +380,18 @@ struct DecodeDev {
   unsigned long long limit_ns;
 };
 
-// The sequence of tiles a CTA walks: its flat row range [lo, hi) of the concatenation over
-// (sequence, head) segments, each segment being the attended rows of one (s, h), cut into tiles of at
-// most TR rows that never cross a segment.
+// The tiles of a worker: its flat row range [x, hi) of the concatenation over (sequence, head)
+// segments, cut into tiles of at most TR rows that never cross a segment.
 struct TileIter {
-  const int64_t* P;
-  int b, H;
-  int64_t hi;
+  int64_t x, hi, Lc, r;
   int s, h;
-  int64_t Lc, r, x;
-  __device__ void init(const int64_t* P_, int b_, int H_, int64_t lo, int64_t hi_) {
-    P = P_;
-    b = b_;
-    H = H_;
-    hi = hi_;
-    int a = 0, z = b - 1;  // largest s with H * P[s] <= lo
-    while (a < z) {
-      const int mid = (a + z + 1) >> 1;
-      if ((int64_t)H * P[mid] <= lo)
-        a = mid;
-      else
-        z = mid - 1;
-    }
-    s = a;
-    Lc = P[s + 1] - P[s];
-    const int64_t o = lo - (int64_t)H * P[s];
-    h = (int)(o / Lc);
-    r = o % Lc;
-    x = lo;
-  }
-  __device__ bool done() const { return x >= hi; }
-  __device__ int n(int TR) const {
+  __device__ __forceinline__ bool done() const { return x >= hi; }
+  __device__ __forceinline__ int n(int TR) const {
     int64_t k = Lc - r;
     if (hi - x < k) k = hi - x;
     return (int)(k < TR ? k : TR);
   }
-  __device__ void advance(int n) {
+  __device__ __forceinline__ void advance(int n, const int64_t* P, int H) {
     x += n;
     r += n;
     if (r == Lc && x < hi) {
@@ -428,86 +407,96 @@ struct TileIter {
   }
 };
 
-__device__ __forceinline__ int cta_of(int64_t x, int64_t R, int G) { return (int)(((x + 1) * G - 1) / R); }
+__device__ __forceinline__ int worker_of(int64_t x, int64_t R, int NW) { return (int)(((x + 1) * NW - 1) / R); }
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
 
 template <typename T, int D>
-__global__ void __launch_bounds__(DecodeCfg<D>::THREADS, 2)
-    decode_kernel(Geometry g, Static st, DecodeDev p) {
+__global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry g, Static st, DecodeDev p) {
   using C = DecodeCfg<D>;
   using L = Lanes<D>;
   extern __shared__ __align__(128) unsigned char smem[];
-  unsigned char* sK = smem;
-  unsigned char* sV = smem + C::S * C::TILE;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + 2 * C::S * C::TILE);
-  uint64_t* empty = full + C::S;
-  float* mo = reinterpret_cast<float*>(empty + C::S);  // [2][NCW][D]
-  float* mml = mo + 2 * C::NCW * D;                     // [2][NCW][2]
-
-  const int cta = blockIdx.x;
-  const int64_t lo = (int64_t)cta * p.R / p.G;
-  const int64_t hi = (int64_t)(cta + 1) * p.R / p.G;
-  if (lo >= hi) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (threadIdx.x == 0) {
+  const int wid = blockIdx.x * C::WARPS + warp;
+  if (wid >= p.NW) return;
+  const int64_t lo = (int64_t)wid * p.R / p.NW;
+  const int64_t hi = (int64_t)(wid + 1) * p.R / p.NW;
+  if (lo >= hi) return;
+
+  unsigned char* base = smem + warp * C::WARP_SMEM;
+  unsigned char* sK = base;                    // [S][TILE]
+  unsigned char* sV = base + C::S * C::TILE;   // [S][TILE]
+  float* qs = reinterpret_cast<float*>(base + 2 * C::S * C::TILE);  // [D]
+  uint64_t* full = reinterpret_cast<uint64_t*>(qs + D);             // [S]
+
+  // stale rows past a tile's end are multiplied by p = 0: start from zeros, never NaN
+  for (int i = lane; i < 2 * C::S * C::TILE / 16; i += 32) reinterpret_cast<uint4*>(base)[i] = make_uint4(0, 0, 0, 0);
+  if (lane == 0) {
 #pragma unroll
-    for (int i = 0; i < C::S; ++i) {
-      mbar_init(&full[i], 1);
-      mbar_init(&empty[i], C::NCW);
-    }
+    for (int i = 0; i < C::S; ++i) mbar_init(&full[i], 1);
     fence_mbar_init();
   }
-  __syncthreads();
+  fence_proxy_async_smem();
+  __syncwarp();
 
-  TileIter it;
-  it.init(p.P, g.b, g.H, lo, hi);
+  // segment holding row `lo`: s = (number of sequences with H*P[s] <= lo) - 1
+  const int H = g.H;
+  int cnt = 0;
+  for (int base_s = 0; base_s < g.b; base_s += 32) {
+    const int k = base_s + lane;
+    const bool le = k < g.b && (int64_t)H * p.P[k] <= lo;
+    cnt += __popc(__ballot_sync(kFull, le));
+  }
+  TileIter ci;  // consumed tiles
+  ci.s = cnt - 1;
+  ci.Lc = p.P[ci.s + 1] - p.P[ci.s];
+  {
+    const int64_t o = lo - (int64_t)H * p.P[ci.s];
+    ci.h = (int)(o / ci.Lc);
+    ci.r = o - (int64_t)ci.h * ci.Lc;
+  }
+  ci.x = lo;
+  ci.hi = hi;
+  TileIter ii = ci;  // issued tiles (lane 0 uses it)
 
-  if (warp == C::NCW) {
-    // ------------------------------- producer -------------------------------
-    if (lane != 0) return;
-    int t = 0;
-    bool ok = true;
-    int cur_s = -1;
-    int64_t seg_base = 0;
-    while (!it.done()) {
-      const int n = it.n(C::TR);
-      const int stage = t % C::S;
-      if (t >= C::S && !mbar_wait_bounded(&empty[stage], ((t / C::S) - 1) & 1, p.limit_ns)) {
-        ok = false;
-        break;
-      }
-      if (it.s != cur_s) {
-        cur_s = it.s;
-        seg_base = st.seq_row0[cur_s] + p.ds[cur_s].begin;
-      }
-      const int64_t row = seg_base + (int64_t)it.h * st.cap[cur_s] + it.r;
-      const uint32_t bytes = (uint32_t)n * L::RB;
-      mbar_arrive_expect_tx(&full[stage], 2 * bytes);
-      bulk_g2s(sK + stage * C::TILE, p.k + row * D, bytes, &full[stage]);
-      bulk_g2s(sV + stage * C::TILE, p.v + row * D, bytes, &full[stage]);
-      it.advance(n);
-      ++t;
+  auto issue = [&](int stage) {
+    const int n = ii.n(C::TR);
+    const DState d = p.ds[ii.s];
+    const int64_t row = st.seq_row0[ii.s] + (int64_t)ii.h * st.cap[ii.s] + d.begin + ii.r;
+    const uint32_t bytes = (uint32_t)n * L::RB;
+    mbar_arrive_expect_tx(&full[stage], 2 * bytes);
+    bulk_g2s(sK + stage * C::TILE, p.k + row * D, bytes, &full[stage]);
+    bulk_g2s(sV + stage * C::TILE, p.v + row * D, bytes, &full[stage]);
+    ii.advance(n, p.P, H);
+  };
+  int issued = 0;
+  if (lane == 0) {
+    while (issued < C::S && !ii.done()) {
+      issue(issued);
+      ++issued;
     }
-    if (!ok) atomicOr(p.status, STATUS_TIMEOUT);
-    // never leave with copies in flight into this CTA's shared memory
-    for (int u = t - C::S < 0 ? 0 : t - C::S; u < t; ++u) mbar_wait_bounded(&full[u % C::S], (u / C::S) & 1, p.limit_ns);
-    return;
   }
 
-  // ------------------------------- consumers -------------------------------
-  const int grp = lane / L::LPR;  // row group within the warp
-  const int tl = lane % L::LPR;   // position within the row
-  float qv[L::EPL], o[L::EPL];
+  const int grp = lane / L::LPR;
+  const int tl = lane % L::LPR;
+  const int rot = (L::A * grp + L::B * tl) % L::NV;
+  float2 qv[L::EPL / 2], o[L::EPL / 2];
   float m = -INFINITY, l = 0.f;
   int64_t mask_lo = 0, mask_hi = 0, begin = 0;
   int cur_s = -1;
-  bool dead = false;  // a bounded wait ran out: keep walking (barriers stay matched) but write nothing
+  bool dead = false;
   bool piece_start = true, piece_whole = false;
-  int piece = 0;
-  int t = 0;
-  while (!it.done()) {
-    const int s = it.s, h = it.h;
-    const int64_t r0 = it.r;
-    const int n = it.n(C::TR);
+  int t = 0;     // tiles consumed
+  int t_ok = 0;  // tiles whose copies were seen complete
+  while (!ci.done()) {
+    const int s = ci.s, h = ci.h;
+    const int64_t r0 = ci.r;
+    const int n = ci.n(C::TR);
     const int stage = t % C::S;
     if (piece_start) {
       if (s != cur_s) {
@@ -517,214 +506,201 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS, 2)
         mask_hi = d.mask_hi;
         begin = d.begin;
       }
-      const uint16_t* qrow = p.q + ((int64_t)s * g.H + h) * D;
+      // stage q (rotated at the query position for RoPE, pre-scaled by scale*log2 e) in natural order
+      const uint16_t* qrow = p.q + ((int64_t)s * H + h) * D;
       const int32_t qpos = p.ds[s].qpos;
       const int half = g.rot / 2;
+      for (int c = lane; c < D; c += 32) {
+        float x = T::f1(qrow[c]);
+        if (c < g.rot) {
+          const bool lo_half = c < half;
+          const float y = T::f1(qrow[lo_half ? c + half : c - half]);
+          float sn, cs;
+          rope_sincos(qpos, st.rope_g[lo_half ? c : c - half], &sn, &cs);
+          x = lo_half ? x * cs - y * sn : x * cs + y * sn;
+        }
+        qs[c] = x * p.qscale;
+      }
+      __syncwarp();
 #pragma unroll
       for (int i = 0; i < L::NV; ++i) {
-#pragma unroll
-        for (int e = 0; e < L::EPV; ++e) {
-          const int c = (tl + L::LPR * i) * L::EPV + e;
-          float x = T::f1(qrow[c]);
-          if (c < g.rot) {
-            const bool lo_half = c < half;
-            const float y = T::f1(qrow[lo_half ? c + half : c - half]);
-            float sn, cs;
-            rope_sincos(qpos, st.rope_g[lo_half ? c : c - half], &sn, &cs);
-            x = lo_half ? x * cs - y * sn : x * cs + y * sn;
-          }
-          qv[i * L::EPV + e] = x * p.qscale;
-          o[i * L::EPV + e] = 0.f;
-        }
+        const int c = tl * L::NV + (i + rot) % L::NV;
+        const float4 a = reinterpret_cast<const float4*>(qs + c * 8)[0];
+        const float4 b = reinterpret_cast<const float4*>(qs + c * 8)[1];
+        qv[i * 4 + 0] = make_float2(a.x, a.y);
+        qv[i * 4 + 1] = make_float2(a.z, a.w);
+        qv[i * 4 + 2] = make_float2(b.x, b.y);
+        qv[i * 4 + 3] = make_float2(b.z, b.w);
       }
+#pragma unroll
+      for (int e = 0; e < L::EPL / 2; ++e) o[e] = make_float2(0.f, 0.f);
       m = -INFINITY;
       l = 0.f;
       piece_whole = (r0 == 0);
       piece_start = false;
     }
-    if (!dead && !mbar_wait_bounded(&full[stage], (t / C::S) & 1, p.limit_ns)) {
-      dead = true;
-      if (lane == 0) atomicOr(p.status, STATUS_TIMEOUT);
-    }
     if (!dead) {
-      const unsigned char* kt = sK + stage * C::TILE;
-      const unsigned char* vt = sV + stage * C::TILE;
+      if (mbar_wait_bounded(&full[stage], (t / C::S) & 1, p.limit_ns)) {
+        t_ok = t + 1;
+      } else {
+        dead = true;
+        if (lane == 0) atomicOr(p.status, STATUS_TIMEOUT);
+      }
+    }
+    const unsigned char* kt = sK + stage * C::TILE;
+    const unsigned char* vt = sV + stage * C::TILE;
+    if (!dead) {
+      // tile-local bounds of the hidden rows
+      const int64_t row0 = begin + r0;
+      int hlo = (int)max((int64_t)0, min((int64_t)C::TR, mask_lo - row0));
+      int hhi = (int)max((int64_t)0, min((int64_t)C::TR, mask_hi - row0));
       float z[C::KPT];
 #pragma unroll
       for (int k = 0; k < C::KPT; ++k) {
-        const int j = (k * C::NCW + warp) * L::RPI + grp;
-        float acc = 0.f;
+        const int j = k * L::RPI + grp;
+        const unsigned char* rowp = kt + j * L::RB;
+        float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
 #pragma unroll
         for (int i = 0; i < L::NV; ++i) {
-          const unsigned char* ptr = kt + j * L::RB + (tl + L::LPR * i) * L::VB;
-          uint32_t w[L::VB / 4];
-          if constexpr (L::VB == 16) {
-            const uint4 u = *reinterpret_cast<const uint4*>(ptr);
-            w[0] = u.x;
-            w[1] = u.y;
-            w[2] = u.z;
-            w[3] = u.w;
-          } else {
-            const uint2 u = *reinterpret_cast<const uint2*>(ptr);
-            w[0] = u.x;
-            w[1] = u.y;
-          }
-#pragma unroll
-          for (int q2 = 0; q2 < L::VB / 4; ++q2) {
-            const float2 f = T::f2(w[q2]);
-            acc = fmaf(qv[i * L::EPV + 2 * q2], f.x, acc);
-            acc = fmaf(qv[i * L::EPV + 2 * q2 + 1], f.y, acc);
-          }
+          const int c = tl * L::NV + (i + rot) % L::NV;
+          const uint4 u = *reinterpret_cast<const uint4*>(rowp + c * 16);
+          acc0 = ffma2(qv[i * 4 + 0], T::f2(u.x), acc0);
+          acc1 = ffma2(qv[i * 4 + 1], T::f2(u.y), acc1);
+          acc0 = ffma2(qv[i * 4 + 2], T::f2(u.z), acc0);
+          acc1 = ffma2(qv[i * 4 + 3], T::f2(u.w), acc1);
         }
+        float zz = (acc0.x + acc1.x) + (acc0.y + acc1.y);
 #pragma unroll
-        for (int off = L::LPR / 2; off >= 1; off >>= 1) acc += __shfl_xor_sync(kFull, acc, off);
-        const int64_t row = begin + r0 + j;
-        const bool valid = j < n && !(row >= mask_lo && row < mask_hi);
-        z[k] = valid ? acc : -INFINITY;
+        for (int off = L::LPR / 2; off >= 1; off >>= 1) zz += __shfl_xor_sync(kFull, zz, off);
+        const bool valid = j < n && (j < hlo || j >= hhi);
+        z[k] = valid ? zz : -INFINITY;
       }
       float mt = z[0];
 #pragma unroll
       for (int k = 1; k < C::KPT; ++k) mt = fmaxf(mt, z[k]);
       const float mn = fmaxf(m, mt);
-      const float alpha = (mn == -INFINITY) ? 1.f : exp2f(m - mn);
+      const float mu = (mn == -INFINITY) ? 0.f : mn;  // every z so far is -inf: keep p = 0, alpha = 0
+      const float alpha = exp2f(m - mu);
       l *= alpha;
+      const float2 a2 = make_float2(alpha, alpha);
 #pragma unroll
-      for (int e = 0; e < L::EPL; ++e) o[e] *= alpha;
+      for (int e = 0; e < L::EPL / 2; ++e) o[e] = fmul2(o[e], a2);
 #pragma unroll
       for (int k = 0; k < C::KPT; ++k) {
-        if (z[k] != -INFINITY) {
-          const int j = (k * C::NCW + warp) * L::RPI + grp;
-          const float pk = exp2f(z[k] - mn);
-          l += pk;
+        const int j = k * L::RPI + grp;
+        const float pk = exp2f(z[k] - mu);
+        l += pk;
+        const float2 p2 = make_float2(pk, pk);
+        const unsigned char* rowp = vt + j * L::RB;
 #pragma unroll
-          for (int i = 0; i < L::NV; ++i) {
-            const unsigned char* ptr = vt + j * L::RB + (tl + L::LPR * i) * L::VB;
-            uint32_t w[L::VB / 4];
-            if constexpr (L::VB == 16) {
-              const uint4 u = *reinterpret_cast<const uint4*>(ptr);
-              w[0] = u.x;
-              w[1] = u.y;
-              w[2] = u.z;
-              w[3] = u.w;
-            } else {
-              const uint2 u = *reinterpret_cast<const uint2*>(ptr);
-              w[0] = u.x;
-              w[1] = u.y;
-            }
-#pragma unroll
-            for (int q2 = 0; q2 < L::VB / 4; ++q2) {
-              const float2 f = T::f2(w[q2]);
-              o[i * L::EPV + 2 * q2] = fmaf(pk, f.x, o[i * L::EPV + 2 * q2]);
-              o[i * L::EPV + 2 * q2 + 1] = fmaf(pk, f.y, o[i * L::EPV + 2 * q2 + 1]);
-            }
-          }
+        for (int i = 0; i < L::NV; ++i) {
+          const int c = tl * L::NV + (i + rot) % L::NV;
+          const uint4 u = *reinterpret_cast<const uint4*>(rowp + c * 16);
+          o[i * 4 + 0] = ffma2(p2, T::f2(u.x), o[i * 4 + 0]);
+          o[i * 4 + 1] = ffma2(p2, T::f2(u.y), o[i * 4 + 1]);
+          o[i * 4 + 2] = ffma2(p2, T::f2(u.z), o[i * 4 + 2]);
+          o[i * 4 + 3] = ffma2(p2, T::f2(u.w), o[i * 4 + 3]);
         }
       }
       m = mn;
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(&empty[stage]);
-    const bool seg_done = (r0 + n == it.Lc);
-    it.advance(n);
+    const bool seg_done = (r0 + n == ci.Lc);
+    ci.advance(n, p.P, H);
     ++t;
-    if (!(seg_done || it.done())) continue;
-
-    // --------------------------- piece end: merge ---------------------------
+    if (seg_done || ci.done()) {
+      // ------------------------- piece end: merge the row groups -------------------------
+      float M = m;
 #pragma unroll
-    for (int off = L::LPR; off < 32; off <<= 1) {
-      const float m2 = __shfl_xor_sync(kFull, m, off);
-      const float l2 = __shfl_xor_sync(kFull, l, off);
-      const float mn = fmaxf(m, m2);
-      const float a1 = (m == -INFINITY) ? 0.f : exp2f(m - mn);
-      const float a2 = (m2 == -INFINITY) ? 0.f : exp2f(m2 - mn);
-      l = l * a1 + l2 * a2;
+      for (int off = 16; off >= 1; off >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, off));
+      const float Mu = (M == -INFINITY) ? 0.f : M;
+      const float e = exp2f(m - Mu);
+      float Ls = l * e;
 #pragma unroll
-      for (int e = 0; e < L::EPL; ++e) o[e] = o[e] * a1 + __shfl_xor_sync(kFull, o[e], off) * a2;
-      m = mn;
-    }
-    const int bsel = piece & 1;
-    float* mo_b = mo + bsel * C::NCW * D;
-    float* ml_b = mml + bsel * C::NCW * 2;
-    if (grp == 0) {
+      for (int off = 16; off >= 1; off >>= 1) Ls += __shfl_xor_sync(kFull, Ls, off);
+      Ls *= 1.0f / (float)L::LPR;  // each row group's l is held by its LPR lanes
+      // scratch: the K buffer of the stage just consumed (its next copy is issued below)
+      float* red = reinterpret_cast<float*>(sK + stage * C::TILE);  // [RPI][D]
+      const float2 e2 = make_float2(e, e);
 #pragma unroll
-      for (int i = 0; i < L::NV; ++i)
-#pragma unroll
-        for (int e = 0; e < L::EPV; ++e) mo_b[warp * D + (tl + L::LPR * i) * L::EPV + e] = o[i * L::EPV + e];
-    }
-    if (lane == 0) {
-      ml_b[warp * 2] = m;
-      ml_b[warp * 2 + 1] = l;
-    }
-    named_bar_sync(1, C::NCW * 32);
-    if (warp == 0 && !dead) {
-      float M = -INFINITY;
-#pragma unroll
-      for (int w = 0; w < C::NCW; ++w) M = fmaxf(M, ml_b[w * 2]);
-      float ew[C::NCW];
-      float Lsum = 0.f;
-#pragma unroll
-      for (int w = 0; w < C::NCW; ++w) {
-        const float mw = ml_b[w * 2];
-        ew[w] = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
-        Lsum += ml_b[w * 2 + 1] * ew[w];
+      for (int i = 0; i < L::NV; ++i) {
+        const int c = tl * L::NV + (i + rot) % L::NV;
+        float4* dst = reinterpret_cast<float4*>(red + grp * D + c * 8);
+        const float2 x0 = fmul2(o[i * 4 + 0], e2), x1 = fmul2(o[i * 4 + 1], e2);
+        const float2 x2 = fmul2(o[i * 4 + 2], e2), x3 = fmul2(o[i * 4 + 3], e2);
+        dst[0] = make_float4(x0.x, x0.y, x1.x, x1.y);
+        dst[1] = make_float4(x2.x, x2.y, x3.x, x3.y);
       }
-      const int seg = s * g.H + h;
-      if (piece_whole && seg_done) {
-        const float inv = 1.f / Lsum;
-        for (int col = lane; col < D; col += 32) {
-          float O = 0.f;
-#pragma unroll
-          for (int w = 0; w < C::NCW; ++w) O += mo_b[w * D + col] * ew[w];
-          p.out[(int64_t)seg * D + col] = O * inv;
-        }
-      } else {
-        float* pp = p.partials + (int64_t)(cta + seg) * (D + 4);
-        for (int col = lane; col < D; col += 32) {
-          float O = 0.f;
-#pragma unroll
-          for (int w = 0; w < C::NCW; ++w) O += mo_b[w * D + col] * ew[w];
-          pp[4 + col] = O;
-        }
-        if (lane == 0) {
-          pp[0] = M;
-          pp[1] = Lsum;
-        }
-        __threadfence();
-        __syncwarp();
-        const int64_t Lc = p.P[s + 1] - p.P[s];
-        const int64_t A = (int64_t)g.H * p.P[s] + (int64_t)h * Lc;
-        const int c_first = cta_of(A, p.R, p.G);
-        const int c_last = cta_of(A + Lc - 1, p.R, p.G);
-        int last = 0;
-        if (lane == 0) last = atomicAdd(&p.counters[seg], 1) == (c_last - c_first);
-        last = __shfl_sync(kFull, last, 0);
-        if (last) {
-          __threadfence();
-          float Mx = -INFINITY;
-          for (int c = c_first; c <= c_last; ++c) Mx = fmaxf(Mx, __ldcg(p.partials + (int64_t)(c + seg) * (D + 4)));
-          float Lx = 0.f;
-          for (int c = c_first; c <= c_last; ++c) {
-            const float* q = p.partials + (int64_t)(c + seg) * (D + 4);
-            const float mc = __ldcg(q);
-            Lx += (mc == -INFINITY) ? 0.f : __ldcg(q + 1) * exp2f(mc - Mx);
-          }
-          const float inv = 1.f / Lx;
+      __syncwarp();
+      const int seg = s * H + h;
+      if (!dead) {
+        if (piece_whole && seg_done) {
+          const float inv = 1.f / Ls;
           for (int col = lane; col < D; col += 32) {
             float O = 0.f;
-            for (int c = c_first; c <= c_last; ++c) {
-              const float* q = p.partials + (int64_t)(c + seg) * (D + 4);
-              const float mc = __ldcg(q);
-              if (mc != -INFINITY) O += __ldcg(q + 4 + col) * exp2f(mc - Mx);
-            }
+#pragma unroll
+            for (int r = 0; r < L::RPI; ++r) O += red[r * D + col];
             p.out[(int64_t)seg * D + col] = O * inv;
           }
-          if (lane == 0) p.counters[seg] = 0;
+        } else {
+          float* pp = p.partials + (int64_t)(wid + seg) * (D + 4);
+          for (int col = lane; col < D; col += 32) {
+            float O = 0.f;
+#pragma unroll
+            for (int r = 0; r < L::RPI; ++r) O += red[r * D + col];
+            pp[4 + col] = O;
+          }
+          if (lane == 0) {
+            pp[0] = M;
+            pp[1] = Ls;
+          }
+          __threadfence();
+          __syncwarp();
+          const int64_t Lc = p.P[s + 1] - p.P[s];
+          const int64_t A = (int64_t)H * p.P[s] + (int64_t)h * Lc;
+          const int w_first = worker_of(A, p.R, p.NW);
+          const int w_last = worker_of(A + Lc - 1, p.R, p.NW);
+          int last = 0;
+          if (lane == 0) last = atomicAdd(&p.counters[seg], 1) == (w_last - w_first);
+          last = __shfl_sync(kFull, last, 0);
+          if (last) {
+            __threadfence();
+            float Mx = -INFINITY;
+            for (int w = w_first; w <= w_last; ++w) Mx = fmaxf(Mx, __ldcg(p.partials + (int64_t)(w + seg) * (D + 4)));
+            const float Mxu = (Mx == -INFINITY) ? 0.f : Mx;
+            float Lx = 0.f;
+            for (int w = w_first; w <= w_last; ++w) {
+              const float* q = p.partials + (int64_t)(w + seg) * (D + 4);
+              Lx += __ldcg(q + 1) * exp2f(__ldcg(q) - Mxu);
+            }
+            const float inv = 1.f / Lx;
+            for (int col = lane; col < D; col += 32) {
+              float O = 0.f;
+              for (int w = w_first; w <= w_last; ++w) {
+                const float* q = p.partials + (int64_t)(w + seg) * (D + 4);
+                O += __ldcg(q + 4 + col) * exp2f(__ldcg(q) - Mxu);
+              }
+              p.out[(int64_t)seg * D + col] = O * inv;
+            }
+            if (lane == 0) p.counters[seg] = 0;
+          }
         }
       }
+      __syncwarp();
+      piece_start = true;
     }
-    ++piece;
-    piece_start = true;
+    // refill the stage just consumed
+    if (lane == 0 && !dead && !ii.done()) {
+      fence_proxy_async_smem();
+      issue(stage);
+      ++issued;
+    }
   }
+  // never leave with copies in flight into this warp's shared memory (only after a timed-out wait)
+  if (lane == 0) {
+    for (int u = t_ok; u < issued; ++u) mbar_wait_bounded(&full[u % C::S], (u / C::S) & 1, p.limit_ns);
+  }
+  __syncwarp();
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -743,11 +719,12 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
     if (e != cudaSuccess) return e;
     occ = o < 1 ? 1 : o;
   }
-  int64_t G = (int64_t)occ * num_sms;
-  const int64_t by_work = (a.R + 2 * C::TR - 1) / (2 * C::TR);
-  if (by_work < G) G = by_work;
-  if (G > kMaxDecodeCtas) G = kMaxDecodeCtas;
-  if (G < 1) G = 1;
+  // one worker per row at most; all resident warps at most
+  int64_t NW = (int64_t)occ * num_sms * C::WARPS;
+  if (a.R < NW) NW = a.R;
+  if (NW > kMaxDecodeWorkers) NW = kMaxDecodeWorkers;
+  if (NW < 1) NW = 1;
+  const int64_t ctas = (NW + C::WARPS - 1) / C::WARPS;
   DecodeDev p;
   const int64_t plane = (int64_t)g.H * g.C * D;
   p.k = buf.k + (int64_t)a.layer * plane;
@@ -755,7 +732,7 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   p.ds = a.dstate;
   p.P = a.P;
   p.R = a.R;
-  p.G = (int)G;
+  p.NW = (int)NW;
   p.q = static_cast<const uint16_t*>(a.q);
   p.out = a.out;
   p.partials = a.partials;
@@ -763,8 +740,8 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   p.status = buf.status;
   p.qscale = a.scale * 1.4426950408889634f;
   p.limit_ns = a.wait_limit_ns;
-  decode_kernel<T, D><<<(unsigned)G, C::THREADS, C::SMEM, stream>>>(g, st, p);
-  *grid = (int)G;
+  decode_kernel<T, D><<<(unsigned)ctas, C::THREADS, C::SMEM, stream>>>(g, st, p);
+  *grid = (int)ctas;
   return cudaGetLastError();
 }
 

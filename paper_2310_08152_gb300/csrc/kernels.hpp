@@ -49,8 +49,8 @@ struct Buffers {
   int* status;
 };
 
-// Largest decode grid; sizes the split-K partial buffer.
-constexpr int kMaxDecodeCtas = 4096;
+// Most decode workers (warps); sizes the split-K partial buffer.
+constexpr int kMaxDecodeWorkers = 8192;
 
 bool dhead_supported(int D);
 
@@ -69,7 +69,7 @@ struct DecodeArgs {
   const void* q;         // [b][H][D]
   float* out;            // [b][H][D]
   float scale;
-  float* partials;       // [(kMaxDecodeCtas + b*H) * (D + 4)]
+  float* partials;       // [(kMaxDecodeWorkers + b*H) * (D + 4)]
   int* counters;         // [b*H], zero between launches
   unsigned long long wait_limit_ns;
 };

@@ -57,7 +57,7 @@ struct WsLayout {
   size_t dyn_bytes = 0;
   size_t dst_map = 0;    // int32 [C]
   size_t counters = 0;   // int32 [b*H]
-  size_t partials = 0;   // float [(kMaxDecodeCtas + b*H) * (D + 4)]
+  size_t partials = 0;   // float [(kMaxDecodeWorkers + b*H) * (D + 4)]
   size_t total = 0;
 };
 
@@ -82,7 +82,7 @@ WsLayout ws_layout(int b, int H, int D, int rot, int64_t C) {
   L.dyn = take(L.dyn_bytes);
   L.dst_map = take(4 * (size_t)C);
   L.counters = take(4 * (size_t)b * H);
-  L.partials = take(4 * (size_t)(kvc::kMaxDecodeCtas + (int64_t)b * H) * (size_t)(D + 4));
+  L.partials = take(4 * (size_t)(kvc::kMaxDecodeWorkers + (int64_t)b * H) * (size_t)(D + 4));
   L.total = o;
   return L;
 }
