@@ -255,8 +255,16 @@ def run_kvc(args, w):
     torch.cuda.synchronize()
     for g in range(args.warmup):
         run.step(inputs[g], out)
-    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(w.M)]
-          for _ in range(args.steps)]
+    # Lean timed loop: device pointers are computed up front and the decode entry point is called
+    # directly, so the host enqueues faster than the GPU drains (no idle gaps from Python overhead).
+    dec = kvc.lib().kvc_decode_attention
+    stream_h = torch.cuda.current_stream().cuda_stream
+    handle = run.cache.handle
+    q_ptrs = [[inputs[g].q[m].data_ptr() for m in range(w.M)] for g in range(steps_total)]
+    out_ptrs = [out[m].data_ptr() for m in range(w.M)]
+    ones = np.ones(w.b, np.int32)
+    # one (start, end) event pair per step around its M decode launches
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     bytes_per_step = []
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
@@ -267,14 +275,18 @@ def run_kvc(args, w):
     clocks.start()
     t_start.record()
     for k in range(args.steps):
+        g = args.warmup + k
+        inp = inputs[g]
+        run.cache.append(inp.kv_k, inp.kv_v, ones, inp.kinds)
         # decode bytes of this step are fixed once the token is appended: computed from the host lengths
-        inp = inputs[args.warmup + k]
-        run.cache.append(inp.kv_k, inp.kv_v, np.ones(w.b, np.int32), inp.kinds)
         bytes_per_step.append(run.decode_bytes())
+        qp = q_ptrs[g]
+        ev[k][0].record()
         for m in range(w.M):
-            ev[k][m][0].record()
-            kvc.kvc_decode_attention(run.cache.handle, m, inp.q[m], w.scale, out[m])
-            ev[k][m][1].record()
+            rc = dec(handle, m, qp[m], w.scale, out_ptrs[m], stream_h)
+            if rc:
+                raise kvc.KvcError(rc, kvc.lib().kvc_last_error().decode())
+        ev[k][1].record()
         seq, cl, cr = run.step_spans(inp.kinds)
         run.g += 1
         if seq:
@@ -290,8 +302,7 @@ def run_kvc(args, w):
         elapsed = float(t.item())
     tokens = w.b * args.steps * world
     value = tokens / elapsed
-    dec_ms = [[ev[k][m][0].elapsed_time(ev[k][m][1]) for m in range(w.M)] for k in range(args.steps)]
-    dec_total_s = sum(sum(r) for r in dec_ms) / 1e3
+    dec_total_s = sum(e0.elapsed_time(e1) for e0, e1 in ev) / 1e3
     dec_bytes_total = sum(b * w.M for b in bytes_per_step)
     achieved = dec_bytes_total / dec_total_s / 1e9
     peak, peak_kind = measured_hbm_peak()

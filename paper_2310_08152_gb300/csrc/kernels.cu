@@ -350,18 +350,27 @@ struct Lanes {
   static_assert(D % 16 == 0 && CH % LPR == 0, "unsupported d_head");
 };
 
+#ifndef KVC_DEC_KPT
+#define KVC_DEC_KPT 2
+#endif
+#ifndef KVC_DEC_STAGES
+#define KVC_DEC_STAGES 3
+#endif
+#ifndef KVC_DEC_WARPS
+#define KVC_DEC_WARPS 4
+#endif
 template <int D>
 struct DecodeCfg {
   using L = Lanes<D>;
-  static constexpr int KPT = 2;                 // rows per lane per tile
+  static constexpr int KPT = KVC_DEC_KPT;       // rows per lane per tile
   static constexpr int TR = KPT * L::RPI;       // rows per tile
   static constexpr int TILE = TR * L::RB;       // bytes per K (or V) tile
-  static constexpr int S = 3;                   // stages per warp
-  static constexpr int WARPS = 4;               // warps per CTA
+  static constexpr int S = KVC_DEC_STAGES;      // stages per warp
+  static constexpr int WARPS = KVC_DEC_WARPS;   // warps per CTA
   static constexpr int THREADS = WARPS * 32;
   static constexpr int WARP_SMEM = (2 * S * TILE + D * 4 + S * 8 + 127) / 128 * 128;
   static constexpr int SMEM = WARPS * WARP_SMEM;
-  static_assert(L::RPI * D * 4 <= TILE, "reduction scratch must fit in one tile");
+  static_assert(L::RPI * D * 4 <= 2 * TILE, "reduction scratch must fit in one stage");
 };
 
 struct DecodeDev {
@@ -378,6 +387,7 @@ struct DecodeDev {
   int* status;
   float qscale;  // scale * log2(e)
   unsigned long long limit_ns;
+  int kv_before_wait;  // the K/V rows may be streamed before the preceding grid completes
 };
 
 // The tiles of a worker: its flat row range [x, hi) of the concatenation over (sequence, head)
@@ -413,6 +423,11 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// Programmatic dependent launch: let the next kernel on the stream be scheduled, and wait for
+// the preceding one (no-ops when the launch did not opt in).
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
 __device__ __forceinline__ float2 fmul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
 
@@ -421,16 +436,23 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
   using C = DecodeCfg<D>;
   using L = Lanes<D>;
   extern __shared__ __align__(128) unsigned char smem[];
+  // The next layer's decode may be scheduled now: its CTAs become resident only as ours retire.
+  pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int wid = blockIdx.x * C::WARPS + warp;
-  if (wid >= p.NW) return;
+  if (wid >= p.NW) {
+    pdl_wait();
+    return;
+  }
   const int64_t lo = (int64_t)wid * p.R / p.NW;
   const int64_t hi = (int64_t)(wid + 1) * p.R / p.NW;
-  if (lo >= hi) return;
+  if (lo >= hi) {
+    pdl_wait();
+    return;
+  }
 
   unsigned char* base = smem + warp * C::WARP_SMEM;
-  unsigned char* sK = base;                    // [S][TILE]
-  unsigned char* sV = base + C::S * C::TILE;   // [S][TILE]
+  unsigned char* stg = base;  // [S][K tile | V tile]
   float* qs = reinterpret_cast<float*>(base + 2 * C::S * C::TILE);  // [D]
   uint64_t* full = reinterpret_cast<uint64_t*>(qs + D);             // [S]
 
@@ -454,27 +476,46 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
   }
   TileIter ci;  // consumed tiles
   ci.s = cnt - 1;
-  ci.Lc = p.P[ci.s + 1] - p.P[ci.s];
+  // everything that depends only on the starting sequence, loaded together
+  const int64_t P0 = p.P[ci.s], P1 = p.P[ci.s + 1];
+  const DState ds0 = p.ds[ci.s];
+  int64_t seg_row0 = st.seq_row0[ci.s];  // issue side: row 0 of (s, h = 0) plus begin
+  int seg_cap = st.cap[ci.s];
+  ci.Lc = P1 - P0;
   {
-    const int64_t o = lo - (int64_t)H * p.P[ci.s];
+    const int64_t o = lo - (int64_t)H * P0;
     ci.h = (int)(o / ci.Lc);
     ci.r = o - (int64_t)ci.h * ci.Lc;
   }
   ci.x = lo;
   ci.hi = hi;
   TileIter ii = ci;  // issued tiles (lane 0 uses it)
+  int seg_s = ci.s;
+  seg_row0 += ds0.begin;
 
   auto issue = [&](int stage) {
     const int n = ii.n(C::TR);
-    const DState d = p.ds[ii.s];
-    const int64_t row = st.seq_row0[ii.s] + (int64_t)ii.h * st.cap[ii.s] + d.begin + ii.r;
+    if (ii.s != seg_s) {
+      seg_s = ii.s;
+      seg_row0 = st.seq_row0[seg_s] + p.ds[seg_s].begin;
+      seg_cap = st.cap[seg_s];
+    }
+    const int64_t row = seg_row0 + (int64_t)ii.h * seg_cap + ii.r;
     const uint32_t bytes = (uint32_t)n * L::RB;
     mbar_arrive_expect_tx(&full[stage], 2 * bytes);
-    bulk_g2s(sK + stage * C::TILE, p.k + row * D, bytes, &full[stage]);
-    bulk_g2s(sV + stage * C::TILE, p.v + row * D, bytes, &full[stage]);
+    bulk_g2s(stg + stage * 2 * C::TILE, p.k + row * D, bytes, &full[stage]);
+    bulk_g2s(stg + stage * 2 * C::TILE + C::TILE, p.v + row * D, bytes, &full[stage]);
     ii.advance(n, p.P, H);
   };
   int issued = 0;
+  // K/V of this layer are not written by the preceding decode: stream them before it completes
+  if (p.kv_before_wait && lane == 0) {
+    while (issued < C::S && !ii.done()) {
+      issue(issued);
+      ++issued;
+    }
+  }
+  pdl_wait();  // q, out and the split-K scratch may be shared with the preceding grid
   if (lane == 0) {
     while (issued < C::S && !ii.done()) {
       issue(issued);
@@ -487,8 +528,9 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
   const int rot = (L::A * grp + L::B * tl) % L::NV;
   float2 qv[L::EPL / 2], o[L::EPL / 2];
   float m = -INFINITY, l = 0.f;
-  int64_t mask_lo = 0, mask_hi = 0, begin = 0;
-  int cur_s = -1;
+  int64_t mask_lo = ds0.mask_lo, mask_hi = ds0.mask_hi, begin = ds0.begin;
+  int32_t qpos = ds0.qpos;
+  int cur_s = ci.s;
   bool dead = false;
   bool piece_start = true, piece_whole = false;
   int t = 0;     // tiles consumed
@@ -505,10 +547,10 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
         mask_lo = d.mask_lo;
         mask_hi = d.mask_hi;
         begin = d.begin;
+        qpos = d.qpos;
       }
       // stage q (rotated at the query position for RoPE, pre-scaled by scale*log2 e) in natural order
       const uint16_t* qrow = p.q + ((int64_t)s * H + h) * D;
-      const int32_t qpos = p.ds[s].qpos;
       const int half = g.rot / 2;
       for (int c = lane; c < D; c += 32) {
         float x = T::f1(qrow[c]);
@@ -547,8 +589,8 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
         if (lane == 0) atomicOr(p.status, STATUS_TIMEOUT);
       }
     }
-    const unsigned char* kt = sK + stage * C::TILE;
-    const unsigned char* vt = sV + stage * C::TILE;
+    const unsigned char* kt = stg + stage * 2 * C::TILE;
+    const unsigned char* vt = kt + C::TILE;
     if (!dead) {
       // tile-local bounds of the hidden rows
       const int64_t row0 = begin + r0;
@@ -619,8 +661,8 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
 #pragma unroll
       for (int off = 16; off >= 1; off >>= 1) Ls += __shfl_xor_sync(kFull, Ls, off);
       Ls *= 1.0f / (float)L::LPR;  // each row group's l is held by its LPR lanes
-      // scratch: the K buffer of the stage just consumed (its next copy is issued below)
-      float* red = reinterpret_cast<float*>(sK + stage * C::TILE);  // [RPI][D]
+      // scratch: the stage just consumed (its next copies are issued below)
+      float* red = reinterpret_cast<float*>(stg + stage * 2 * C::TILE);  // [RPI][D]
       const float2 e2 = make_float2(e, e);
 #pragma unroll
       for (int i = 0; i < L::NV; ++i) {
@@ -665,19 +707,25 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
           last = __shfl_sync(kFull, last, 0);
           if (last) {
             __threadfence();
+            // lane k holds part w_first + k (parts of one segment are few; loop for more than 32)
+            const int np = w_last - w_first + 1;
             float Mx = -INFINITY;
-            for (int w = w_first; w <= w_last; ++w) Mx = fmaxf(Mx, __ldcg(p.partials + (int64_t)(w + seg) * (D + 4)));
+            for (int k = lane; k < np; k += 32) Mx = fmaxf(Mx, __ldcg(p.partials + (int64_t)(w_first + k + seg) * (D + 4)));
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) Mx = fmaxf(Mx, __shfl_xor_sync(kFull, Mx, off));
             const float Mxu = (Mx == -INFINITY) ? 0.f : Mx;
             float Lx = 0.f;
-            for (int w = w_first; w <= w_last; ++w) {
-              const float* q = p.partials + (int64_t)(w + seg) * (D + 4);
+            for (int k = lane; k < np; k += 32) {
+              const float* q = p.partials + (int64_t)(w_first + k + seg) * (D + 4);
               Lx += __ldcg(q + 1) * exp2f(__ldcg(q) - Mxu);
             }
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) Lx += __shfl_xor_sync(kFull, Lx, off);
             const float inv = 1.f / Lx;
             for (int col = lane; col < D; col += 32) {
               float O = 0.f;
-              for (int w = w_first; w <= w_last; ++w) {
-                const float* q = p.partials + (int64_t)(w + seg) * (D + 4);
+              for (int k = 0; k < np; ++k) {
+                const float* q = p.partials + (int64_t)(w_first + k + seg) * (D + 4);
                 O += __ldcg(q + 4 + col) * exp2f(__ldcg(q) - Mxu);
               }
               p.out[(int64_t)seg * D + col] = O * inv;
@@ -740,9 +788,20 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   p.status = buf.status;
   p.qscale = a.scale * 1.4426950408889634f;
   p.limit_ns = a.wait_limit_ns;
-  decode_kernel<T, D><<<(unsigned)ctas, C::THREADS, C::SMEM, stream>>>(g, st, p);
+  p.kv_before_wait = a.kv_before_wait;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)ctas);
+  cfg.blockDim = dim3(C::THREADS);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, decode_kernel<T, D>, g, st, p);
   *grid = (int)ctas;
-  return cudaGetLastError();
+  return e;
 }
 
 template <typename T, int D>

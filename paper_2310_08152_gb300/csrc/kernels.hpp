@@ -72,6 +72,9 @@ struct DecodeArgs {
   float* partials;       // [(kMaxDecodeWorkers + b*H) * (D + 4)]
   int* counters;         // [b*H], zero between launches
   unsigned long long wait_limit_ns;
+  // 1 when the kernel launched before this one on the stream was a decode (which writes no K/V):
+  // K/V tiles are then requested before that kernel has completed (programmatic dependent launch).
+  int kv_before_wait;
 };
 
 // Returns the grid used through *grid (0 if nothing launched).

@@ -207,6 +207,8 @@ struct kvc_cache {
   std::string decode_err;
   int64_t R = 0;
   int64_t launches = 0;
+  // the last kernel this cache launched was a decode (it writes no K/V rows)
+  bool last_was_decode = false;
 
   kvc_cache(const kvc_config& c, int64_t C_) : cfg(c), C(C_), bk(c.b, (kvc::Policy)c.policy, c.seq_capacity) {
     cap.assign(c.seq_capacity, c.seq_capacity + c.b);
@@ -560,6 +562,7 @@ kvc_status kvc_append(kvc_cache* c, int layer, const void* k, const void* v, con
     cudaError_t e = kvc::launch_append(g, c->stat(), c->bufs(), plan, c->batch_ntok, m0, nl, m0 == 0, k, v, stream);
     if (e != cudaSuccess) return cuda_fail(e, "append kernel");
     c->launches += 1;
+    c->last_was_decode = false;
   }
   c->layers_done = m0 + nl;
   return ok();
@@ -620,6 +623,7 @@ kvc_status kvc_compress_spans(kvc_cache* c, const int32_t* seq, const int64_t* c
                           reinterpret_cast<const int32_t*>(c->wsp(c->ws.dyn + c->ws.dyn_payload + aff_bytes)),
                           reinterpret_cast<int32_t*>(c->wsp(c->ws.dst_map)), stream, &launched);
   c->launches += launched;
+  c->last_was_decode = false;
   if (e != cudaSuccess) return cuda_fail(e, "compaction kernels");
   return ok();
 }
@@ -647,10 +651,12 @@ kvc_status kvc_decode_attention(kvc_cache* c, int layer, const void* q, float sc
   a.partials = reinterpret_cast<float*>(c->wsp(c->ws.partials));
   a.counters = reinterpret_cast<int*>(c->wsp(c->ws.counters));
   a.wait_limit_ns = 2000000000ull;
+  a.kv_before_wait = c->last_was_decode ? 1 : 0;
   int grid = 0;
   cudaError_t e = kvc::launch_decode(c->geom(), c->stat(), c->bufs(), a, c->num_sms, stream, &grid);
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel");
   c->launches += grid > 0 ? 1 : 0;
+  c->last_was_decode = true;
   return ok();
 }
 
