@@ -351,13 +351,13 @@ struct Lanes {
 };
 
 #ifndef KVC_DEC_KPT
-#define KVC_DEC_KPT 2
+#define KVC_DEC_KPT 4
 #endif
 #ifndef KVC_DEC_STAGES
 #define KVC_DEC_STAGES 3
 #endif
 #ifndef KVC_DEC_WARPS
-#define KVC_DEC_WARPS 4
+#define KVC_DEC_WARPS 1
 #endif
 template <int D>
 struct DecodeCfg {
@@ -388,6 +388,7 @@ struct DecodeDev {
   float qscale;  // scale * log2(e)
   unsigned long long limit_ns;
   int kv_before_wait;  // the K/V rows may be streamed before the preceding grid completes
+  int seg_per_worker;  // 1: worker w owns segment w whole; 0: stream-K split of the rows
 };
 
 // The tiles of a worker: its flat row range [x, hi) of the concatenation over (sequence, head)
@@ -444,8 +445,17 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
     pdl_wait();
     return;
   }
-  const int64_t lo = (int64_t)wid * p.R / p.NW;
-  const int64_t hi = (int64_t)(wid + 1) * p.R / p.NW;
+  const int H = g.H;
+  int64_t lo, hi;
+  if (p.seg_per_worker) {  // segment wid = (s, h) whole
+    const int s0 = wid / H;
+    const int64_t a = p.P[s0], z = p.P[s0 + 1];
+    lo = (int64_t)H * a + (int64_t)(wid % H) * (z - a);
+    hi = lo + (z - a);
+  } else {
+    lo = (int64_t)wid * p.R / p.NW;
+    hi = (int64_t)(wid + 1) * p.R / p.NW;
+  }
   if (lo >= hi) {
     pdl_wait();
     return;
@@ -467,12 +477,15 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
   __syncwarp();
 
   // segment holding row `lo`: s = (number of sequences with H*P[s] <= lo) - 1
-  const int H = g.H;
   int cnt = 0;
-  for (int base_s = 0; base_s < g.b; base_s += 32) {
-    const int k = base_s + lane;
-    const bool le = k < g.b && (int64_t)H * p.P[k] <= lo;
-    cnt += __popc(__ballot_sync(kFull, le));
+  if (p.seg_per_worker) {
+    cnt = wid / H + 1;
+  } else {
+    for (int base_s = 0; base_s < g.b; base_s += 32) {
+      const int k = base_s + lane;
+      const bool le = k < g.b && (int64_t)H * p.P[k] <= lo;
+      cnt += __popc(__ballot_sync(kFull, le));
+    }
   }
   TileIter ci;  // consumed tiles
   ci.s = cnt - 1;
@@ -767,9 +780,15 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
     if (e != cudaSuccess) return e;
     occ = o < 1 ? 1 : o;
   }
-  // one worker per row at most; all resident warps at most
-  int64_t NW = (int64_t)occ * num_sms * C::WARPS;
-  if (a.R < NW) NW = a.R;
+  // One wave of resident warps.  When every (sequence, head) segment fits in that wave and the
+  // longest is within 1.3x of the mean, each warp takes one segment whole (no split-K partials);
+  // otherwise the rows are split evenly over the resident warps (stream-K).
+  const int64_t resident = (int64_t)occ * num_sms * C::WARPS;
+  const int64_t nseg = (int64_t)g.b * g.H;
+  const bool by_segment = a.n_segments > 0 && nseg <= resident && nseg <= kMaxDecodeWorkers &&
+                          10 * a.max_segment * a.n_segments <= 13 * a.R;
+  int64_t NW = by_segment ? nseg : resident;
+  if (!by_segment && a.R < NW) NW = a.R;
   if (NW > kMaxDecodeWorkers) NW = kMaxDecodeWorkers;
   if (NW < 1) NW = 1;
   const int64_t ctas = (NW + C::WARPS - 1) / C::WARPS;
@@ -789,6 +808,7 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   p.qscale = a.scale * 1.4426950408889634f;
   p.limit_ns = a.wait_limit_ns;
   p.kv_before_wait = a.kv_before_wait;
+  p.seg_per_worker = by_segment ? 1 : 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)ctas);
   cfg.blockDim = dim3(C::THREADS);

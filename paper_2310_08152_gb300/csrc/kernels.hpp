@@ -75,6 +75,9 @@ struct DecodeArgs {
   // 1 when the kernel launched before this one on the stream was a decode (which writes no K/V):
   // K/V tiles are then requested before that kernel has completed (programmatic dependent launch).
   int kv_before_wait;
+  // segment statistics of the uploaded state: segments with rows, and the longest one
+  int64_t n_segments;
+  int64_t max_segment;
 };
 
 // Returns the grid used through *grid (0 if nothing launched).

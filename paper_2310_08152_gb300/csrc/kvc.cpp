@@ -206,6 +206,7 @@ struct kvc_cache {
   bool decode_ok = false;
   std::string decode_err;
   int64_t R = 0;
+  int64_t n_segments = 0, max_segment = 0;
   int64_t launches = 0;
   // the last kernel this cache launched was a decode (it writes no K/V rows)
   bool last_was_decode = false;
@@ -304,6 +305,8 @@ struct kvc_cache {
     decode_ok = true;
     decode_err.clear();
     P[0] = 0;
+    n_segments = 0;
+    max_segment = 0;
     for (int s = 0; s < cfg.b; ++s) {
       kvc::DecodeView v;
       std::string err;
@@ -323,6 +326,10 @@ struct kvc_cache {
         decode_ok = false;
       }
       P[s + 1] = P[s] + Lc;
+      if (Lc > 0) {
+        n_segments += cfg.H;
+        max_segment = std::max(max_segment, Lc);
+      }
     }
     R = (int64_t)cfg.H * P[cfg.b];
   }
@@ -652,6 +659,8 @@ kvc_status kvc_decode_attention(kvc_cache* c, int layer, const void* q, float sc
   a.counters = reinterpret_cast<int*>(c->wsp(c->ws.counters));
   a.wait_limit_ns = 2000000000ull;
   a.kv_before_wait = c->last_was_decode ? 1 : 0;
+  a.n_segments = c->n_segments;
+  a.max_segment = c->max_segment;
   int grid = 0;
   cudaError_t e = kvc::launch_decode(c->geom(), c->stat(), c->bufs(), a, c->num_sms, stream, &grid);
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel");
