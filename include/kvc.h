@@ -186,6 +186,23 @@ kvc_status kvc_compress_spans(kvc_cache* cache, const int32_t* seq, const int64_
  * Split-K over the kept rows with a log-sum-exp combine; reads only the kept rows. */
 kvc_status kvc_decode_attention(kvc_cache* cache, int layer, const void* q, float scale, float* out, void* stream);
 
+/* The same decode as kvc_decode_attention, for callers that cannot allocate device memory at run
+ * time (for example code running inside a fixed memory pool, or under an allocator that forbids
+ * new device allocations): its split-K scratch -- partial results and arrival counters -- lives in
+ * a file-scope __device__ array of libkvc instead of the cache workspace, so the call allocates
+ * nothing (no cudaMalloc or cudaFree, no allocating library routine).  The paper has no counterpart;
+ * this is an interface convenience.
+ *   - Size limit: 8 MiB, enough while 4*((8192 + b*H)*(d_head + 4) rounded up to 256) + 4*b*H fits;
+ *     larger caches get KVC_ERR_UNSUPPORTED (use kvc_decode_attention).
+ *   - Every GPU that loads the library holds the 8 MiB until the process exits.
+ *   - The first call on a device looks up the array's device address (cudaGetSymbolAddress); make
+ *     that first call before any stream capture.
+ *   - All calls share the one array: calls that overlap on the GPU (different streams, caches or
+ *     threads without ordering between them) race and give wrong results.  Each call clears the
+ *     counters it relies on before its kernel runs, on `stream`. */
+kvc_status kvc_decode_attention_static_scratch(kvc_cache* cache, int layer, const void* q, float scale, float* out,
+                                               void* stream);
+
 /* Verification (synchronous: waits for `stream`): the history of `seq` and the mask for its next
  * query as in kvc_book_layout, with the stored rows read back from the device metadata
  * (stored_orig_idx, stored_pos, n_stored = the device's view).  Buffers of `cap` entries. */

@@ -245,6 +245,12 @@ def kvc_decode_attention(cache: int, layer: int, q, scale: float, out, stream=No
     _check(lib().kvc_decode_attention(cache, layer, _ptr(q), float(scale), _ptr(out), _stream_handle(stream)))
 
 
+def kvc_decode_attention_static_scratch(cache: int, layer: int, q, scale: float, out, stream=None):
+    """Decode whose split-K scratch is the library's static device array (no allocation anywhere)."""
+    _check(lib().kvc_decode_attention_static_scratch(cache, layer, _ptr(q), float(scale), _ptr(out),
+                                                     _stream_handle(stream)))
+
+
 def kvc_masked_reference_layout(cache: int, seq: int, cap: int, stream=None):
     kind = np.empty(cap, np.uint8)
     pos = np.empty(cap, np.int32)

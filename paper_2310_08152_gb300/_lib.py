@@ -51,6 +51,7 @@ SIGNATURES = [
     ("kvc_append", c_int, [P, c_int, P, P, P, P, P, P]),
     ("kvc_compress_spans", c_int, [P, P, P, P, c_int, P]),
     ("kvc_decode_attention", c_int, [P, c_int, P, c_float, P, P]),
+    ("kvc_decode_attention_static_scratch", c_int, [P, c_int, P, c_float, P, P]),
     ("kvc_masked_reference_layout", c_int, [P, c_int, c_int64, P, P, P, P, P, P, P, P]),
     ("kvc_device_status", c_int, [P, P, P]),
     ("kvc_launch_count", c_int64, [P]),

@@ -20,6 +20,7 @@
 
 #include <cmath>
 #include <cstdint>
+#include <mutex>
 
 #include "kernels.hpp"
 
@@ -899,6 +900,36 @@ cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& bu
     if (g.dtype == 1) return launch_decode_t<BF16T, D>(g, st, buf, a, num_sms, stream, grid);
     return launch_decode_t<F16T, D>(g, st, buf, a, num_sms, stream, grid);
   });
+}
+
+// ---------------------------------------------------------------------------------------------
+// Split-K scratch without allocation.  Every GPU that loads this library holds the array until the
+// process exits; all calls share it (kvc_decode_attention_static_scratch documents the contract).
+// In host code `g_decode_static_scratch` names a host-side stand-in: only the address returned by
+// cudaGetSymbolAddress may be handed to a kernel.
+// ---------------------------------------------------------------------------------------------
+__device__ __align__(256) unsigned char g_decode_static_scratch[kStaticDecodeScratchBytes];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_static_scratch_mu;
+void* g_static_scratch_addr[kMaxDevices] = {};
+}  // namespace
+
+cudaError_t static_decode_scratch(void** ptr) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_static_scratch_mu);
+  if (g_static_scratch_addr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_decode_static_scratch);
+    if (e != cudaSuccess) return e;
+    g_static_scratch_addr[dev] = p;
+  }
+  *ptr = g_static_scratch_addr[dev];
+  return cudaSuccess;
 }
 
 }  // namespace kvc

@@ -84,4 +84,10 @@ struct DecodeArgs {
 cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a,
                           int num_sms, cudaStream_t stream, int* grid);
 
+// Split-K scratch in a file-scope device array (kernels.cu), for callers that cannot allocate
+// device memory.  *ptr gets its device address on the current device; the address is looked up
+// with cudaGetSymbolAddress the first time a device asks for it.
+constexpr size_t kStaticDecodeScratchBytes = size_t(8) << 20;
+cudaError_t static_decode_scratch(void** ptr);
+
 }  // namespace kvc

@@ -669,6 +669,57 @@ kvc_status kvc_decode_attention(kvc_cache* c, int layer, const void* q, float sc
   return ok();
 }
 
+kvc_status kvc_decode_attention_static_scratch(kvc_cache* c, int layer, const void* q, float scale, float* out,
+                                               void* stream_) {
+  if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  if (layer < 0 || layer >= c->cfg.M) return fail(KVC_ERR_INVALID_ARG, "layer %d out of range", layer);
+  if (!q || !out) return fail(KVC_ERR_INVALID_ARG, "q/out are NULL");
+  if (!std::isfinite(scale)) return fail(KVC_ERR_INVALID_ARG, "scale is not finite");
+  if (layer >= c->layers_done) return fail(KVC_ERR_STATE, "layer %d of the last tokens is not written yet", layer);
+  if (!c->cuda_ready) return fail(KVC_ERR_STATE, "nothing appended yet");
+  if (!c->decode_ok) return fail(KVC_ERR_STATE, "%s", c->decode_err.c_str());
+  if (c->R <= 0) return fail(KVC_ERR_STATE, "no sequence has a token to query");
+  // split-K partials for every possible worker and segment, then one arrival counter per segment
+  const size_t segs = (size_t)c->cfg.b * c->cfg.H;
+  const size_t part_bytes = align_up(4 * ((size_t)kvc::kMaxDecodeWorkers + segs) * (size_t)(c->cfg.d_head + 4), 256);
+  const size_t need = part_bytes + 4 * segs;
+  if (need > kvc::kStaticDecodeScratchBytes)
+    return fail(KVC_ERR_UNSUPPORTED,
+                "b*H=%zu with d_head=%d needs %zu bytes of split-K scratch; the static array holds %zu "
+                "(use kvc_decode_attention with the cache workspace)",
+                segs, c->cfg.d_head, need, kvc::kStaticDecodeScratchBytes);
+  kvc_status st = c->ensure_cuda(stream);
+  if (st != KVC_OK) return st;
+  void* scratch = nullptr;
+  cudaError_t e = kvc::static_decode_scratch(&scratch);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress (static decode scratch)");
+  int* counters = reinterpret_cast<int*>(static_cast<unsigned char*>(scratch) + part_bytes);
+  // the array keeps the previous call's contents: the arrival counters must start from zero
+  e = cudaMemsetAsync(counters, 0, 4 * segs, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync (static decode scratch)");
+  kvc::DecodeArgs a;
+  a.layer = layer;
+  a.dstate = reinterpret_cast<const kvc::DState*>(c->wsp(c->ws.dyn));
+  a.P = reinterpret_cast<const int64_t*>(c->wsp(c->ws.dyn + c->ws.dyn_P));
+  a.R = c->R;
+  a.q = q;
+  a.out = out;
+  a.scale = scale;
+  a.partials = static_cast<float*>(scratch);
+  a.counters = counters;
+  a.wait_limit_ns = 2000000000ull;
+  a.kv_before_wait = 0;
+  a.n_segments = c->n_segments;
+  a.max_segment = c->max_segment;
+  int grid = 0;
+  e = kvc::launch_decode(c->geom(), c->stat(), c->bufs(), a, c->num_sms, stream, &grid);
+  if (e != cudaSuccess) return cuda_fail(e, "decode kernel (static scratch)");
+  c->launches += grid > 0 ? 1 : 0;
+  c->last_was_decode = true;
+  return ok();
+}
+
 kvc_status kvc_masked_reference_layout(kvc_cache* c, int seq, int64_t cap, uint8_t* kind_full, int32_t* pos_full,
                                        uint8_t* visible_full, int64_t* n_full, int32_t* stored_orig_idx,
                                        int32_t* stored_pos, int64_t* n_stored, void* stream_) {
