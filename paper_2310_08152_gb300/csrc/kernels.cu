@@ -351,23 +351,29 @@ struct Lanes {
   static_assert(D % 16 == 0 && CH % LPR == 0, "unsupported d_head");
 };
 
-#ifndef KVC_DEC_KPT
-#define KVC_DEC_KPT 4
+// Two shapes of the per-warp pipeline.  One warp per segment runs few warps, each of which must
+// keep many bytes in flight: 4 rows per lane per tile (64-row tiles at d=64), 3 stages.  Stream-K
+// runs a full wave of warps: 2 rows per lane per tile, 3 stages, so that more warps fit per SM.
+#ifndef KVC_DEC_SEG_KPT
+#define KVC_DEC_SEG_KPT 4
 #endif
-#ifndef KVC_DEC_STAGES
-#define KVC_DEC_STAGES 3
+#ifndef KVC_DEC_SEG_STAGES
+#define KVC_DEC_SEG_STAGES 3
 #endif
-#ifndef KVC_DEC_WARPS
-#define KVC_DEC_WARPS 1
+#ifndef KVC_DEC_STREAM_KPT
+#define KVC_DEC_STREAM_KPT 2
 #endif
-template <int D>
+#ifndef KVC_DEC_STREAM_STAGES
+#define KVC_DEC_STREAM_STAGES 3
+#endif
+template <int D, int KPT_, int S_>
 struct DecodeCfg {
   using L = Lanes<D>;
-  static constexpr int KPT = KVC_DEC_KPT;       // rows per lane per tile
+  static constexpr int KPT = KPT_;              // rows per lane per tile
   static constexpr int TR = KPT * L::RPI;       // rows per tile
   static constexpr int TILE = TR * L::RB;       // bytes per K (or V) tile
-  static constexpr int S = KVC_DEC_STAGES;      // stages per warp
-  static constexpr int WARPS = KVC_DEC_WARPS;   // warps per CTA
+  static constexpr int S = S_;                  // stages per warp
+  static constexpr int WARPS = 1;               // warps per CTA
   static constexpr int THREADS = WARPS * 32;
   static constexpr int WARP_SMEM = (2 * S * TILE + D * 4 + S * 8 + 127) / 128 * 128;
   static constexpr int SMEM = WARPS * WARP_SMEM;
@@ -433,9 +439,9 @@ __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;"
 __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
 __device__ __forceinline__ float2 fmul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
 
-template <typename T, int D>
-__global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry g, Static st, DecodeDev p) {
-  using C = DecodeCfg<D>;
+template <typename T, int D, int KPT, int S>
+__global__ void __launch_bounds__(32) decode_kernel(Geometry g, Static st, DecodeDev p) {
+  using C = DecodeCfg<D, KPT, S>;
   using L = Lanes<D>;
   extern __shared__ __align__(128) unsigned char smem[];
   // The next layer's decode may be scheduled now: its CTAs become resident only as ours retire.
@@ -537,6 +543,25 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
     }
   }
 
+  // raw q of the next piece (and its rotation partner), fetched one tile ahead of its use
+  constexpr int QPL = (D + 31) / 32;
+  float qa[QPL], qb[QPL];
+  auto fetch_q = [&](int s_, int h_) {
+    const uint16_t* qrow = p.q + ((int64_t)s_ * H + h_) * D;
+    const int half = g.rot / 2;
+#pragma unroll
+    for (int j = 0; j < QPL; ++j) {
+      const int c = lane + 32 * j;
+      qa[j] = 0.f;
+      qb[j] = 0.f;
+      if (c < D) {
+        qa[j] = T::f1(qrow[c]);
+        if (c < g.rot) qb[j] = T::f1(qrow[c < half ? c + half : c - half]);
+      }
+    }
+  };
+  fetch_q(ci.s, ci.h);
+  DState dn = ds0;
   const int grp = lane / L::LPR;
   const int tl = lane % L::LPR;
   const int rot = (L::A * grp + L::B * tl) % L::NV;
@@ -555,27 +580,28 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
     const int n = ci.n(C::TR);
     const int stage = t % C::S;
     if (piece_start) {
-      if (s != cur_s) {
+      if (s != cur_s) {  // the next sequence's state was prefetched with its q
         cur_s = s;
-        const DState d = p.ds[s];
-        mask_lo = d.mask_lo;
-        mask_hi = d.mask_hi;
-        begin = d.begin;
-        qpos = d.qpos;
+        mask_lo = dn.mask_lo;
+        mask_hi = dn.mask_hi;
+        begin = dn.begin;
+        qpos = dn.qpos;
       }
       // stage q (rotated at the query position for RoPE, pre-scaled by scale*log2 e) in natural order
-      const uint16_t* qrow = p.q + ((int64_t)s * H + h) * D;
       const int half = g.rot / 2;
-      for (int c = lane; c < D; c += 32) {
-        float x = T::f1(qrow[c]);
-        if (c < g.rot) {
-          const bool lo_half = c < half;
-          const float y = T::f1(qrow[lo_half ? c + half : c - half]);
-          float sn, cs;
-          rope_sincos(qpos, st.rope_g[lo_half ? c : c - half], &sn, &cs);
-          x = lo_half ? x * cs - y * sn : x * cs + y * sn;
+#pragma unroll
+      for (int j = 0; j < QPL; ++j) {
+        const int c = lane + 32 * j;
+        if (c < D) {
+          float x = qa[j];
+          if (c < g.rot) {
+            const bool lo_half = c < half;
+            float sn, cs;
+            rope_sincos(qpos, st.rope_g[lo_half ? c : c - half], &sn, &cs);
+            x = lo_half ? x * cs - qb[j] * sn : x * cs + qb[j] * sn;
+          }
+          qs[c] = x * p.qscale;
         }
-        qs[c] = x * p.qscale;
       }
       __syncwarp();
 #pragma unroll
@@ -594,6 +620,12 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
       l = 0.f;
       piece_whole = (r0 == 0);
       piece_start = false;
+    }
+    if (r0 + n == ci.Lc && ci.x + n < ci.hi) {  // this tile ends the segment: fetch the next piece's q
+      TileIter nx = ci;
+      nx.advance(n, p.P, H);
+      fetch_q(nx.s, nx.h);
+      if (nx.s != s) dn = p.ds[nx.s];
     }
     if (!dead) {
       if (mbar_wait_bounded(&full[stage], (t / C::S) & 1, p.limit_ns)) {
@@ -768,31 +800,34 @@ __global__ void __launch_bounds__(DecodeCfg<D>::THREADS) decode_kernel(Geometry 
 // ---------------------------------------------------------------------------------------------
 // dispatch
 // ---------------------------------------------------------------------------------------------
-template <typename T, int D>
-cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a, int num_sms,
-                            cudaStream_t stream, int* grid) {
-  using C = DecodeCfg<D>;
-  static int occ = -1;
-  if (occ < 0) {
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+// Resident CTAs per SM of one kernel instance, per device (the shared-memory attribute is set on
+// each device the first time the instance runs there).
+template <typename T, int D, int KPT, int S>
+cudaError_t decode_occupancy(int* occ_out) {
+  using C = DecodeCfg<D, KPT, S>;
+  static std::mutex mu;
+  static int occ[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (occ[dev] == 0) {
+    e = cudaFuncSetAttribute(decode_kernel<T, D, KPT, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     int o = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, decode_kernel<T, D>, C::THREADS, C::SMEM);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, decode_kernel<T, D, KPT, S>, C::THREADS, C::SMEM);
     if (e != cudaSuccess) return e;
-    occ = o < 1 ? 1 : o;
+    occ[dev] = o < 1 ? 1 : o;
   }
-  // One wave of resident warps.  When every (sequence, head) segment fits in that wave and the
-  // longest is within 1.3x of the mean, each warp takes one segment whole (no split-K partials);
-  // otherwise the rows are split evenly over the resident warps (stream-K).
-  const int64_t resident = (int64_t)occ * num_sms * C::WARPS;
-  const int64_t nseg = (int64_t)g.b * g.H;
-  const bool by_segment = a.n_segments > 0 && nseg <= resident && nseg <= kMaxDecodeWorkers &&
-                          10 * a.max_segment * a.n_segments <= 13 * a.R;
-  int64_t NW = by_segment ? nseg : resident;
-  if (!by_segment && a.R < NW) NW = a.R;
-  if (NW > kMaxDecodeWorkers) NW = kMaxDecodeWorkers;
-  if (NW < 1) NW = 1;
-  const int64_t ctas = (NW + C::WARPS - 1) / C::WARPS;
+  *occ_out = occ[dev];
+  return cudaSuccess;
+}
+
+template <typename T, int D, int KPT, int S>
+cudaError_t launch_decode_cfg(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a,
+                              int64_t NW, bool by_segment, cudaStream_t stream, int* grid) {
+  using C = DecodeCfg<D, KPT, S>;
   DecodeDev p;
   const int64_t plane = (int64_t)g.H * g.C * D;
   p.k = buf.k + (int64_t)a.layer * plane;
@@ -810,6 +845,7 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   p.limit_ns = a.wait_limit_ns;
   p.kv_before_wait = a.kv_before_wait;
   p.seg_per_worker = by_segment ? 1 : 0;
+  const int64_t ctas = (NW + C::WARPS - 1) / C::WARPS;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)ctas);
   cfg.blockDim = dim3(C::THREADS);
@@ -820,9 +856,33 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, decode_kernel<T, D>, g, st, p);
   *grid = (int)ctas;
-  return e;
+  return cudaLaunchKernelEx(&cfg, decode_kernel<T, D, KPT, S>, g, st, p);
+}
+
+template <typename T, int D>
+cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a, int num_sms,
+                            cudaStream_t stream, int* grid) {
+  constexpr int SK = KVC_DEC_SEG_KPT, SS = KVC_DEC_SEG_STAGES;
+  constexpr int TK = KVC_DEC_STREAM_KPT, TS = KVC_DEC_STREAM_STAGES;
+  // One warp per (sequence, head) segment when all segments fit one wave of resident warps and the
+  // longest is within 1.3x of the mean: no split-K partials.  Otherwise the rows are split evenly
+  // over a full wave of warps (stream-K).
+  int occ_seg = 0;
+  cudaError_t e = decode_occupancy<T, D, SK, SS>(&occ_seg);
+  if (e != cudaSuccess) return e;
+  const int64_t nseg = (int64_t)g.b * g.H;
+  const bool by_segment = a.n_segments > 0 && nseg <= (int64_t)occ_seg * num_sms && nseg <= kMaxDecodeWorkers &&
+                          10 * a.max_segment * a.n_segments <= 13 * a.R;
+  if (by_segment) return launch_decode_cfg<T, D, SK, SS>(g, st, buf, a, nseg, true, stream, grid);
+  int occ = 0;
+  e = decode_occupancy<T, D, TK, TS>(&occ);
+  if (e != cudaSuccess) return e;
+  int64_t NW = (int64_t)occ * num_sms;
+  if (a.R < NW) NW = a.R;
+  if (NW > kMaxDecodeWorkers) NW = kMaxDecodeWorkers;
+  if (NW < 1) NW = 1;
+  return launch_decode_cfg<T, D, TK, TS>(g, st, buf, a, NW, false, stream, grid);
 }
 
 template <typename T, int D>
