@@ -440,7 +440,7 @@ __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return _
 __device__ __forceinline__ float2 fmul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
 
 template <typename T, int D, int KPT, int S>
-__global__ void __launch_bounds__(32) decode_kernel(Geometry g, Static st, DecodeDev p) {
+__global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, DecodeDev p) {
   using C = DecodeCfg<D, KPT, S>;
   using L = Lanes<D>;
   extern __shared__ __align__(128) unsigned char smem[];
