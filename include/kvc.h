@@ -218,6 +218,13 @@ kvc_status kvc_device_status(kvc_cache* cache, void* stream, int32_t* word);
 /* Number of kernels this cache has launched so far. */
 int64_t kvc_launch_count(const kvc_cache* cache);
 
+/* How the last decode launch divided its work (host-side record, no synchronisation):
+ * plan[0] = mode (0: the kept rows split evenly over a full wave of warps, split (sequence, head)
+ * segments merged by a log-sum-exp combine; 1 / 2: one warp per segment with the wide / narrow
+ * shared-memory pipeline; -1: nothing launched yet), plan[1] = warps, plan[2] = rows per tile,
+ * plan[3] = pipeline stages per warp. */
+kvc_status kvc_last_decode_plan(const kvc_cache* cache, int32_t* plan);
+
 #ifdef __cplusplus
 }
 #endif

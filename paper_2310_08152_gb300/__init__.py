@@ -275,6 +275,12 @@ def kvc_launch_count(cache: int) -> int:
     return lib().kvc_launch_count(cache)
 
 
+def kvc_last_decode_plan(cache: int) -> dict:
+    a = np.zeros(4, np.int32)
+    _check(lib().kvc_last_decode_plan(cache, a.ctypes.data))
+    return {"mode": int(a[0]), "workers": int(a[1]), "tile_rows": int(a[2]), "stages": int(a[3])}
+
+
 class KVCache:
     """A sentinel-compressed KV cache: owns its device buffers (torch) and the library handle."""
 
@@ -360,6 +366,10 @@ class KVCache:
     @property
     def launch_count(self) -> int:
         return kvc_launch_count(self.handle)
+
+    @property
+    def last_decode_plan(self) -> dict:
+        return kvc_last_decode_plan(self.handle)
 
     def close(self):
         if getattr(self, "handle", None):

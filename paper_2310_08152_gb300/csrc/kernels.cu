@@ -351,20 +351,26 @@ struct Lanes {
   static_assert(D % 16 == 0 && CH % LPR == 0, "unsupported d_head");
 };
 
-// Two shapes of the per-warp pipeline.  One warp per segment runs few warps, each of which must
-// keep many bytes in flight: 4 rows per lane per tile (64-row tiles at d=64), 3 stages.  Stream-K
-// runs a full wave of warps: 2 rows per lane per tile, 3 stages, so that more warps fit per SM.
+// Shapes of the per-warp pipeline (rows per lane per tile x stages).  One warp per segment wants
+// the largest in-flight window that still lets every segment have a resident warp: 4x3 (64-row
+// tiles at d=64), else 2x3.  Stream-K runs a full wave of warps: 2x2 fits the most warps per SM.
 #ifndef KVC_DEC_SEG_KPT
 #define KVC_DEC_SEG_KPT 4
 #endif
 #ifndef KVC_DEC_SEG_STAGES
 #define KVC_DEC_SEG_STAGES 3
 #endif
+#ifndef KVC_DEC_SEG2_KPT
+#define KVC_DEC_SEG2_KPT 2
+#endif
+#ifndef KVC_DEC_SEG2_STAGES
+#define KVC_DEC_SEG2_STAGES 3
+#endif
 #ifndef KVC_DEC_STREAM_KPT
 #define KVC_DEC_STREAM_KPT 2
 #endif
 #ifndef KVC_DEC_STREAM_STAGES
-#define KVC_DEC_STREAM_STAGES 3
+#define KVC_DEC_STREAM_STAGES 2
 #endif
 template <int D, int KPT_, int S_>
 struct DecodeCfg {
@@ -862,19 +868,31 @@ cudaError_t launch_decode_cfg(const Geometry& g, const Static& st, const Buffers
 
 template <typename T, int D>
 cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a, int num_sms,
-                            cudaStream_t stream, int* grid) {
-  constexpr int SK = KVC_DEC_SEG_KPT, SS = KVC_DEC_SEG_STAGES;
+                            cudaStream_t stream, int* grid, DecodePlan* plan) {
+  constexpr int AK = KVC_DEC_SEG_KPT, AS = KVC_DEC_SEG_STAGES;
+  constexpr int BK = KVC_DEC_SEG2_KPT, BS = KVC_DEC_SEG2_STAGES;
   constexpr int TK = KVC_DEC_STREAM_KPT, TS = KVC_DEC_STREAM_STAGES;
-  // One warp per (sequence, head) segment when all segments fit one wave of resident warps and the
-  // longest is within 1.3x of the mean: no split-K partials.  Otherwise the rows are split evenly
-  // over a full wave of warps (stream-K).
-  int occ_seg = 0;
-  cudaError_t e = decode_occupancy<T, D, SK, SS>(&occ_seg);
-  if (e != cudaSuccess) return e;
+  // One warp per (sequence, head) segment when the segments are balanced (longest within 1.3x of
+  // the mean) and all fit one wave of resident warps: no split-K partials.  The wider pipeline
+  // shape is tried first.  Otherwise the rows are split evenly over a full wave (stream-K).
   const int64_t nseg = (int64_t)g.b * g.H;
-  const bool by_segment = a.n_segments > 0 && nseg <= (int64_t)occ_seg * num_sms && nseg <= kMaxDecodeWorkers &&
-                          10 * a.max_segment * a.n_segments <= 13 * a.R;
-  if (by_segment) return launch_decode_cfg<T, D, SK, SS>(g, st, buf, a, nseg, true, stream, grid);
+  const bool balanced = a.n_segments > 0 && nseg <= kMaxDecodeWorkers && 10 * a.max_segment * a.n_segments <= 13 * a.R;
+  cudaError_t e;
+  if (balanced) {
+    int occ = 0;
+    e = decode_occupancy<T, D, AK, AS>(&occ);
+    if (e != cudaSuccess) return e;
+    if (nseg <= (int64_t)occ * num_sms) {
+      *plan = {1, (int)nseg, AK * Lanes<D>::RPI, AS};
+      return launch_decode_cfg<T, D, AK, AS>(g, st, buf, a, nseg, true, stream, grid);
+    }
+    e = decode_occupancy<T, D, BK, BS>(&occ);
+    if (e != cudaSuccess) return e;
+    if (nseg <= (int64_t)occ * num_sms) {
+      *plan = {2, (int)nseg, BK * Lanes<D>::RPI, BS};
+      return launch_decode_cfg<T, D, BK, BS>(g, st, buf, a, nseg, true, stream, grid);
+    }
+  }
   int occ = 0;
   e = decode_occupancy<T, D, TK, TS>(&occ);
   if (e != cudaSuccess) return e;
@@ -882,6 +900,7 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   if (a.R < NW) NW = a.R;
   if (NW > kMaxDecodeWorkers) NW = kMaxDecodeWorkers;
   if (NW < 1) NW = 1;
+  *plan = {0, (int)NW, TK * Lanes<D>::RPI, TS};
   return launch_decode_cfg<T, D, TK, TS>(g, st, buf, a, NW, false, stream, grid);
 }
 
@@ -952,13 +971,14 @@ cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& b
 }
 
 cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a, int num_sms,
-                          cudaStream_t stream, int* grid) {
+                          cudaStream_t stream, int* grid, DecodePlan* plan) {
   *grid = 0;
+  *plan = {-1, 0, 0, 0};
   if (a.R <= 0) return cudaSuccess;
   return by_dhead(g.D, [&](auto dc) {
     constexpr int D = decltype(dc)::value;
-    if (g.dtype == 1) return launch_decode_t<BF16T, D>(g, st, buf, a, num_sms, stream, grid);
-    return launch_decode_t<F16T, D>(g, st, buf, a, num_sms, stream, grid);
+    if (g.dtype == 1) return launch_decode_t<BF16T, D>(g, st, buf, a, num_sms, stream, grid, plan);
+    return launch_decode_t<F16T, D>(g, st, buf, a, num_sms, stream, grid, plan);
   });
 }
 

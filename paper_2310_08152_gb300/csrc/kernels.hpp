@@ -80,9 +80,15 @@ struct DecodeArgs {
   int64_t max_segment;
 };
 
-// Returns the grid used through *grid (0 if nothing launched).
+// How a decode launch split its work: mode 0 = stream-K over all rows, 1 / 2 = one warp per
+// (sequence, head) segment with the wide / narrow pipeline; workers = warps; tile rows; stages.
+struct DecodePlan {
+  int mode, workers, tile_rows, stages;
+};
+
+// Returns the grid used through *grid (0 if nothing launched) and the plan through *plan.
 cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a,
-                          int num_sms, cudaStream_t stream, int* grid);
+                          int num_sms, cudaStream_t stream, int* grid, DecodePlan* plan);
 
 // Split-K scratch in a file-scope device array (kernels.cu), for callers that cannot allocate
 // device memory.  *ptr gets its device address on the current device; the address is looked up

@@ -210,6 +210,7 @@ struct kvc_cache {
   int64_t launches = 0;
   // the last kernel this cache launched was a decode (it writes no K/V rows)
   bool last_was_decode = false;
+  kvc::DecodePlan last_plan{-1, 0, 0, 0};
 
   kvc_cache(const kvc_config& c, int64_t C_) : cfg(c), C(C_), bk(c.b, (kvc::Policy)c.policy, c.seq_capacity) {
     cap.assign(c.seq_capacity, c.seq_capacity + c.b);
@@ -662,7 +663,7 @@ kvc_status kvc_decode_attention(kvc_cache* c, int layer, const void* q, float sc
   a.n_segments = c->n_segments;
   a.max_segment = c->max_segment;
   int grid = 0;
-  cudaError_t e = kvc::launch_decode(c->geom(), c->stat(), c->bufs(), a, c->num_sms, stream, &grid);
+  cudaError_t e = kvc::launch_decode(c->geom(), c->stat(), c->bufs(), a, c->num_sms, stream, &grid, &c->last_plan);
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel");
   c->launches += grid > 0 ? 1 : 0;
   c->last_was_decode = true;
@@ -713,7 +714,7 @@ kvc_status kvc_decode_attention_static_scratch(kvc_cache* c, int layer, const vo
   a.n_segments = c->n_segments;
   a.max_segment = c->max_segment;
   int grid = 0;
-  e = kvc::launch_decode(c->geom(), c->stat(), c->bufs(), a, c->num_sms, stream, &grid);
+  e = kvc::launch_decode(c->geom(), c->stat(), c->bufs(), a, c->num_sms, stream, &grid, &c->last_plan);
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel (static scratch)");
   c->launches += grid > 0 ? 1 : 0;
   c->last_was_decode = true;
@@ -764,5 +765,14 @@ kvc_status kvc_device_status(kvc_cache* c, void* stream_, int32_t* word) {
 }
 
 int64_t kvc_launch_count(const kvc_cache* c) { return c ? c->launches : 0; }
+
+kvc_status kvc_last_decode_plan(const kvc_cache* c, int32_t* plan) {
+  if (!c || !plan) return fail(KVC_ERR_INVALID_ARG, "NULL argument");
+  plan[0] = c->last_plan.mode;
+  plan[1] = c->last_plan.workers;
+  plan[2] = c->last_plan.tile_rows;
+  plan[3] = c->last_plan.stages;
+  return ok();
+}
 
 }  // extern "C"
