@@ -295,6 +295,46 @@ def workload_config(w):
             "l2": "inputs larger than L2 (every step reads GBs of distinct K/V rows)"}
 
 
+def aggregate(local_tokens: int, local_elapsed: float, device=None):
+    """Whole-job tokens (sum over ranks) and elapsed time (max over ranks); identity on one rank."""
+    import torch
+    import torch.distributed as dist
+
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return local_tokens, local_elapsed
+    t = torch.tensor([float(local_elapsed)], dtype=torch.float64, device=device)
+    n = torch.tensor([float(local_tokens)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    return int(n.item()), float(t.item())
+
+
+def time_prompt_compaction(run, w):
+    """Frees every prompt span in one go (one compaction over all sequences and layers) and reports
+    the row-move bandwidth: bytes = 2 (read + write) x moved rows x row bytes x M x 2 (K, V) x H."""
+    import torch
+
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record()
+    run.compress_prompt()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    ln = run.cache.lengths()[0]
+    moved = 0
+    for s in range(w.b):
+        if w.prompt_spans[s]:
+            first = min(a for a, _ in w.prompt_spans[s])  # first dropped row: nothing before it moves
+            moved += int(ln[s]) - first
+    nbytes = 2 * moved * w.d * 2 * w.M * 2 * w.H
+    peak, kind = measured_hbm_peak()
+    gbs = nbytes / (ms * 1e-3) / 1e9 if ms > 0 else None
+    return {"kernels": "compact_scan_kernel + compact_move_kernel", "moved_rows_per_stream": moved,
+            "bytes": nbytes, "ms": ms, "achieved": gbs, "peak": peak, "unit": "GB/s",
+            "frac": (gbs / peak) if gbs else None, "peak_kind": kind}
+
+
 def run_kvc(args, w):
     import torch
     import torch.distributed as dist
@@ -311,7 +351,8 @@ def run_kvc(args, w):
 
     # ---------------- device-resident run ----------------
     run = harness.Runner(w, steps_total, device=dev)
-    run.load_prompt()
+    run.load_prompt(compress=False)
+    compaction = time_prompt_compaction(run, w)
     inputs = [run.make_step_inputs(g) for g in range(steps_total)]
     out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device=dev)
     torch.cuda.synchronize()
@@ -358,12 +399,9 @@ def run_kvc(args, w):
     clk = clocks.stop()
     launches = run.cache.launch_count - launches0
     elapsed = t_start.elapsed_time(t_end) / 1e3
-    if world > 1:
-        t = torch.tensor([elapsed], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed = float(t.item())
-    tokens = w.b * args.steps * world
+    tokens, elapsed = aggregate(w.b * args.steps, elapsed, dev)
     value = tokens / elapsed
+    plan = run.cache.last_decode_plan
     dec_total_s = sum(e0.elapsed_time(e1) for e0, e1 in ev) / 1e3
     dec_bytes_total = sum(b * w.M for b in bytes_per_step)
     achieved = dec_bytes_total / dec_total_s / 1e9
@@ -391,7 +429,11 @@ def run_kvc(args, w):
                          "traffic": recorded_traffic(w.name),
                          "bytes_per_launch_mean": dec_bytes_total / launches_decode,
                          "launch_us_mean": dec_total_s / launches_decode * 1e6},
+            "decode_plan": {"mode": ["stream-K", "warp per segment (wide)", "warp per segment (narrow)"][plan["mode"]]
+                            if plan["mode"] >= 0 else None, "warps": plan["workers"],
+                            "tile_rows": plan["tile_rows"], "stages": plan["stages"]},
             "decode_share_of_step": dec_total_s / elapsed,
+            "compaction": compaction,
             "gpu_launches": launches,
             "device_status": status,
             "clocks": clk,
@@ -448,14 +490,10 @@ def run_e2e(args, w, dev, world):
         one(args.warmup + k)
     torch.cuda.synchronize()
     elapsed = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([elapsed], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed = float(t.item())
+    tokens, elapsed = aggregate(w.b * args.steps, elapsed, dev)
     del run
     torch.cuda.empty_cache()
-    return {"value": w.b * args.steps * world / elapsed, "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h}
+    return {"value": tokens / elapsed, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
 
 def main():
