@@ -157,6 +157,16 @@ def opt13b(b: int = 16, L: int = 2048, M: int = 24) -> Workload:
                          "generated: <CL> at g%33==0, <CR> at g%33==32")
 
 
+def opt13b_uncompressed(b: int = 16, L: int = 2048, M: int = 24) -> Workload:
+    """The OPT-1.3B-shaped cache with no sentinel spans (r = 0): every token is kept.  Used as the
+    reference point for DRAM traffic scaling with the compressed length."""
+    kinds = np.zeros(L, dtype=np.uint8)
+    return Workload("opt1.3b_r0", 1, M=M, H=32, d=64, dtype="f16", b=b, prompt_kinds=[kinds.copy() for _ in range(b)],
+                    prompt_spans=[[] for _ in range(b)], n_steps=128, gen_kind=_normal_gen,
+                    scale=1.0 / math.sqrt(64), seed=SEED_BASE + 1,
+                    note=f"OPT-1.3B-shaped, no spans (r=0): M={M}, H=32, d=64, fp16, b={b}, L={L}")
+
+
 def opt27b(b: int = 32, L: int = 4096, M: int = 32) -> Workload:
     kinds, spans = block_kinds(L, 44)
     return Workload("opt2.7b", 2, M=M, H=32, d=80, dtype="bf16", b=b, prompt_kinds=[kinds.copy() for _ in range(b)],
@@ -205,7 +215,8 @@ def ragged(b: int = 128, lmin: int = 256, lmax: int = 8192, M: int = 24, steps: 
 
 
 def by_name(name: str, **kw) -> Workload:
-    table = {"tiny": tiny, "opt1.3b": opt13b, "opt2.7b": opt27b, "ragged": ragged}
+    table = {"tiny": tiny, "opt1.3b": opt13b, "opt1.3b_r0": opt13b_uncompressed, "opt2.7b": opt27b,
+             "ragged": ragged}
     if name.startswith("rope3b"):
         interior = int(name.split("_I")[1]) if "_I" in name else 32
         return rope3b(interior=interior, **kw)
