@@ -1,8 +1,8 @@
 // sm_103a kernels of the sentinel-compressed KV decode path.
 //
 //   append_kernel         new tokens' K/V rows into the ragged cache (+ RoPE on K, + metadata)
-//   compact_scan_kernel   keep flags -> warp-ballot/popc + block exclusive scan -> destination map,
-//                         in-place move of the position / history-index metadata
+//   compact_scan_kernel   keep flags -> warp-ballot/popc + block exclusive scan -> source row of every
+//                         destination row, in-place move of the position / history-index metadata
 //   compact_move_kernel   in-place, ascending, 16-byte vectorised row moves of every
 //                         (layer, K/V, head) stream of the affected sequences
 //   decode_kernel         split-K single-query attention over the kept rows: every warp is a worker
@@ -101,6 +101,10 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
     if ((it & 63u) == 0 && global_ns() - t0 > limit_ns) return false;
   }
 }
+// Programmatic dependent launch: let the next kernel on the stream be scheduled, and wait for
+// the preceding one (no-ops when the launch did not opt in).
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
   asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                    smem_addr(dst)),
@@ -202,15 +206,16 @@ __device__ __forceinline__ bool in_ranges(int32_t o, const int2* rg, int nr) {
 __global__ void __launch_bounds__(kScanThreads) compact_scan_kernel(Static st, Buffers buf,
                                                                     const AffSeq* __restrict__ aff,
                                                                     const int2* __restrict__ ranges,
-                                                                    int32_t* __restrict__ dst_map) {
+                                                                    int32_t* __restrict__ src_map) {
   __shared__ int2 srg[kMaxSmemRanges];
   __shared__ int wsum[32];
   __shared__ int total;
+  pdl_launch_dependents();  // the row-move kernel may be scheduled; it waits for this grid's results
   const AffSeq a = aff[blockIdx.x];
   const int64_t off = st.off[a.s];
   int32_t* pos = buf.pos + off;
   int32_t* orig = buf.orig + off;
-  int32_t* dmap = dst_map + off;
+  int32_t* smap = src_map + off;  // smap[dst] = source row of the row that lands at dst
   const int nr = a.n_ranges;
   const int2* rg = ranges + a.range_off;
   if (nr <= kMaxSmemRanges) {
@@ -247,8 +252,8 @@ __global__ void __launch_bounds__(kScanThreads) compact_scan_kernel(Static st, B
     }
     __syncthreads();
     const int dst = base + wsum[warp] + pre;
-    if (valid) dmap[i] = keep ? dst : -1;
     if (keep) {  // dst <= i: lands on rows already read (this chunk, after the barrier) or earlier chunks
+      smap[dst] = i;
       orig[dst] = o;
       pos[dst] = p;
     }
@@ -259,10 +264,11 @@ __global__ void __launch_bounds__(kScanThreads) compact_scan_kernel(Static st, B
 }
 
 // ---------------------------------------------------------------------------------------------
-// a4: row moves.  One CTA owns one (sequence, layer, K/V, head) stream and walks 128-row chunks
-// upward.  Every kept row moves down (dst < src), so stores of chunk k land below chunk k+1's
-// sources: the loads of chunk k+1 are issued before storing chunk k, and a barrier separates
-// each chunk's loads from its own stores.
+// a4: row moves.  One CTA owns one (sequence, layer, K/V, head) stream and walks its DESTINATION
+// rows upward in chunks of 128, so every chunk moves 128 full rows however sparse the kept rows
+// are.  A kept row only moves down (source >= destination): the stores of chunk k land below every
+// source of chunk k+1, so chunk k+1's loads are issued before chunk k's stores, and a barrier
+// separates each chunk's loads from its own stores.
 // ---------------------------------------------------------------------------------------------
 constexpr int kMoveThreads = 256;
 constexpr int kMoveRows = 128;
@@ -270,10 +276,11 @@ constexpr int kMoveRows = 128;
 template <int D>
 __global__ void __launch_bounds__(kMoveThreads) compact_move_kernel(Geometry g, Static st, Buffers buf,
                                                                     const AffSeq* __restrict__ aff,
-                                                                    const int32_t* __restrict__ dst_map) {
+                                                                    const int32_t* __restrict__ src_map) {
   constexpr int VPR = D / 8;                                  // 16-byte vectors per row
   constexpr int U = kMoveRows * VPR / kMoveThreads;           // vectors per thread per chunk
   static_assert(kMoveRows * VPR % kMoveThreads == 0, "chunk must split evenly");
+  pdl_wait();  // the source map and the plan come from the scan kernel
   const int streams = g.M * 2 * g.H;
   const int ai = blockIdx.x / streams;
   const int sidx = blockIdx.x % streams;
@@ -284,33 +291,31 @@ __global__ void __launch_bounds__(kMoveThreads) compact_move_kernel(Geometry g, 
   uint16_t* plane = kv ? buf.v : buf.k;
   uint4* base = reinterpret_cast<uint4*>(
       plane + ((int64_t)m * g.H * g.C + st.seq_row0[a.s] + (int64_t)h * st.cap[a.s]) * D);
-  const int32_t* dmap = dst_map + st.off[a.s];
+  const int32_t* smap = src_map + st.off[a.s];
 
   uint4 ra[U], rb[U];
   int da[U], db[U];
-  auto load = [&](int r0, uint4* reg, int* dv) {
+  auto load = [&](int d0, uint4* reg, int* dv) {
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int vi = threadIdx.x + u * kMoveThreads;
-      const int row = r0 + vi / VPR;
+      const int row = d0 + vi / VPR;  // destination row
       const int col = vi % VPR;
       int d = -1;
-      if (row < a.len_old) {
-        const int dr = __ldg(dmap + row);
-        if (dr >= 0) {
-          reg[u] = base[(int64_t)row * VPR + col];
-          d = dr * VPR + col;
-        }
+      if (row < a.len_new) {
+        const int src = __ldg(smap + row);
+        reg[u] = base[(int64_t)src * VPR + col];
+        d = row * VPR + col;
       }
       dv[u] = d;
     }
   };
-  int r0 = a.first_row;
-  if (r0 >= a.len_old) return;
-  load(r0, ra, da);
-  for (; r0 < a.len_old; r0 += kMoveRows) {
-    const bool more = r0 + kMoveRows < a.len_old;
-    if (more) load(r0 + kMoveRows, rb, db);
+  int d0 = a.first_row;
+  if (d0 >= a.len_new) return;
+  load(d0, ra, da);
+  for (; d0 < a.len_new; d0 += kMoveRows) {
+    const bool more = d0 + kMoveRows < a.len_new;
+    if (more) load(d0 + kMoveRows, rb, db);
     __syncthreads();
 #pragma unroll
     for (int u = 0; u < U; ++u)
@@ -437,10 +442,6 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// Programmatic dependent launch: let the next kernel on the stream be scheduled, and wait for
-// the preceding one (no-ops when the launch did not opt in).
-__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
 __device__ __forceinline__ float2 fmul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
@@ -952,19 +953,28 @@ cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& bu
 }
 
 cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& buf, const AffSeq* aff, int n_aff,
-                           const int32_t* ranges, int32_t* dst_map, cudaStream_t stream, int* launched) {
+                           const int32_t* ranges, int32_t* src_map, cudaStream_t stream, int* launched) {
   *launched = 0;
   if (n_aff <= 0) return cudaSuccess;
   compact_scan_kernel<<<n_aff, kScanThreads, 0, stream>>>(st, buf, aff, reinterpret_cast<const int2*>(ranges),
-                                                         dst_map);
+                                                         src_map);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   *launched = 1;
   const int64_t blocks = (int64_t)n_aff * g.M * 2 * g.H;
   e = by_dhead(g.D, [&](auto dc) {
     constexpr int D = decltype(dc)::value;
-    compact_move_kernel<D><<<(unsigned)blocks, kMoveThreads, 0, stream>>>(g, st, buf, aff, dst_map);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks);
+    cfg.blockDim = dim3(kMoveThreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, compact_move_kernel<D>, g, st, buf, aff, (const int32_t*)src_map);
   });
   if (e == cudaSuccess) *launched = 2;
   return e;

@@ -59,7 +59,7 @@ cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& bu
                           cudaStream_t stream);
 
 cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& buf, const AffSeq* aff, int n_aff,
-                           const int32_t* ranges, int32_t* dst_map, cudaStream_t stream, int* launched);
+                           const int32_t* ranges, int32_t* src_map, cudaStream_t stream, int* launched);
 
 struct DecodeArgs {
   int layer;

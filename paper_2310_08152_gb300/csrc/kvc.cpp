@@ -55,7 +55,7 @@ struct WsLayout {
   size_t dyn_P = 0;      // offset of P inside dyn
   size_t dyn_payload = 0;  // offset of the payload inside dyn
   size_t dyn_bytes = 0;
-  size_t dst_map = 0;    // int32 [C]
+  size_t src_map = 0;    // int32 [C]: source row of each destination row of a compaction
   size_t counters = 0;   // int32 [b*H]
   size_t partials = 0;   // float [(kMaxDecodeWorkers + b*H) * (D + 4)]
   size_t total = 0;
@@ -80,7 +80,7 @@ WsLayout ws_layout(int b, int H, int D, int rot, int64_t C) {
   const size_t cmp = sizeof(kvc::AffSeq) * (size_t)b + 8 * (size_t)(C / 2 + 1);
   L.dyn_bytes = L.dyn_payload + std::max(tok, cmp);
   L.dyn = take(L.dyn_bytes);
-  L.dst_map = take(4 * (size_t)C);
+  L.src_map = take(4 * (size_t)C);
   L.counters = take(4 * (size_t)b * H);
   L.partials = take(4 * (size_t)(kvc::kMaxDecodeWorkers + (int64_t)b * H) * (size_t)(D + 4));
   L.total = o;
@@ -629,7 +629,7 @@ kvc_status kvc_compress_spans(kvc_cache* c, const int32_t* seq, const int64_t* c
   e = kvc::launch_compact(c->geom(), c->stat(), c->bufs(),
                           reinterpret_cast<const kvc::AffSeq*>(c->wsp(c->ws.dyn + c->ws.dyn_payload)), n_aff,
                           reinterpret_cast<const int32_t*>(c->wsp(c->ws.dyn + c->ws.dyn_payload + aff_bytes)),
-                          reinterpret_cast<int32_t*>(c->wsp(c->ws.dst_map)), stream, &launched);
+                          reinterpret_cast<int32_t*>(c->wsp(c->ws.src_map)), stream, &launched);
   c->launches += launched;
   c->last_was_decode = false;
   if (e != cudaSuccess) return cuda_fail(e, "compaction kernels");
