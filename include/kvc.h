@@ -215,6 +215,12 @@ kvc_status kvc_masked_reference_layout(kvc_cache* cache, int seq, int64_t cap, u
  * KVC_ERR_TIMEOUT or KVC_ERR_DEVICE_CHECK accordingly. */
 kvc_status kvc_device_status(kvc_cache* cache, void* stream, int32_t* word);
 
+/* Checks the kernels' failure reporting without a fault: launches one warp that waits, with the
+ * same bounded wait the decode kernel uses, on a barrier phase that nothing completes.  After
+ * limit_ns (0 < limit_ns <= 2e9) the wait gives up and sets the timeout bit of the status word, so
+ * that the next kvc_device_status returns KVC_ERR_TIMEOUT; the context stays usable.  Asynchronous. */
+kvc_status kvc_check_bounded_wait(kvc_cache* cache, uint64_t limit_ns, void* stream);
+
 /* Number of kernels this cache has launched so far. */
 int64_t kvc_launch_count(const kvc_cache* cache);
 

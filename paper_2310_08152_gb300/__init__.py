@@ -271,6 +271,10 @@ def kvc_device_status(cache: int, stream=None) -> int:
     return w.value
 
 
+def kvc_check_bounded_wait(cache: int, limit_ns: int, stream=None):
+    _check(lib().kvc_check_bounded_wait(cache, int(limit_ns), _stream_handle(stream)))
+
+
 def kvc_launch_count(cache: int) -> int:
     return lib().kvc_launch_count(cache)
 

@@ -55,6 +55,7 @@ SIGNATURES = [
     ("kvc_masked_reference_layout", c_int, [P, c_int, c_int64, P, P, P, P, P, P, P, P]),
     ("kvc_device_status", c_int, [P, P, P]),
     ("kvc_launch_count", c_int64, [P]),
+    ("kvc_check_bounded_wait", c_int, [P, ctypes.c_uint64, P]),
     ("kvc_last_decode_plan", c_int, [P, P]),
 ]
 

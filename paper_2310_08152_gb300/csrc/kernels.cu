@@ -993,6 +993,28 @@ cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& bu
 }
 
 // ---------------------------------------------------------------------------------------------
+// Timeout path check: one warp waits, with the decode's bounded wait, on an mbarrier phase that
+// nothing completes; when the limit runs out it records STATUS_TIMEOUT like a decode would.
+// ---------------------------------------------------------------------------------------------
+namespace {
+__global__ void bounded_wait_check_kernel(int* status, unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+  if (!mbar_wait_bounded(&bar, 0, limit_ns) && threadIdx.x == 0) atomicOr(status, STATUS_TIMEOUT);
+  __syncwarp();
+}
+}  // namespace
+
+cudaError_t launch_bounded_wait_check(int* status, unsigned long long limit_ns, cudaStream_t stream) {
+  bounded_wait_check_kernel<<<1, 32, 0, stream>>>(status, limit_ns);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------------------------
 // Split-K scratch without allocation.  Every GPU that loads this library holds the array until the
 // process exits; all calls share it (kvc_decode_attention_static_scratch documents the contract).
 // In host code `g_decode_static_scratch` names a host-side stand-in: only the address returned by

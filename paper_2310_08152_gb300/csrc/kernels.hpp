@@ -90,6 +90,10 @@ struct DecodePlan {
 cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a,
                           int num_sms, cudaStream_t stream, int* grid, DecodePlan* plan);
 
+// One warp waits on an mbarrier phase that never completes, with the limit given; the bounded wait
+// gives up and sets STATUS_TIMEOUT in *status.  Exercises the kernels' timeout reporting.
+cudaError_t launch_bounded_wait_check(int* status, unsigned long long limit_ns, cudaStream_t stream);
+
 // Split-K scratch in a file-scope device array (kernels.cu), for callers that cannot allocate
 // device memory.  *ptr gets its device address on the current device; the address is looked up
 // with cudaGetSymbolAddress the first time a device asks for it.

@@ -764,6 +764,20 @@ kvc_status kvc_device_status(kvc_cache* c, void* stream_, int32_t* word) {
   return fail(KVC_ERR_DEVICE_CHECK, "a kernel's consistency check failed (status 0x%x)", w);
 }
 
+kvc_status kvc_check_bounded_wait(kvc_cache* c, uint64_t limit_ns, void* stream_) {
+  if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
+  if (limit_ns == 0 || limit_ns > 2000000000ull)
+    return fail(KVC_ERR_INVALID_ARG, "limit_ns=%llu must be in (0, 2e9]", (unsigned long long)limit_ns);
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  kvc_status st = c->ensure_cuda(stream);
+  if (st != KVC_OK) return st;
+  cudaError_t e = kvc::launch_bounded_wait_check(reinterpret_cast<int*>(c->wsp(c->ws.hdr)), limit_ns, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "bounded-wait check kernel");
+  c->launches += 1;
+  c->last_was_decode = false;
+  return ok();
+}
+
 int64_t kvc_launch_count(const kvc_cache* c) { return c ? c->launches : 0; }
 
 kvc_status kvc_last_decode_plan(const kvc_cache* c, int32_t* plan) {

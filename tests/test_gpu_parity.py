@@ -221,3 +221,23 @@ def test_every_scheduling_mode(name, w, mode):
     run, _ = run_workload(w, steps=2, check_steps={0, 1}, seqs=None)
     plan = run.cache.last_decode_plan
     assert plan["mode"] == mode, plan
+
+
+def test_bounded_wait_reports_timeout_and_context_survives():
+    # a wait that nothing completes must give up, report KVC_ERR_TIMEOUT and leave the GPU usable
+    w = wl.tiny()
+    run = harness.Runner(w, steps=1)
+    run.load_prompt()
+    assert run.cache.device_status() == 0
+    kvc.kvc_check_bounded_wait(run.cache.handle, 2_000_000)  # 2 ms
+    with pytest.raises(kvc.KvcError) as e:
+        run.cache.device_status()
+    assert e.value.status == 8
+    assert run.cache.device_status() == 0  # read and cleared
+    out = torch.empty(1, 2, 4, 64, device="cuda")
+    inp = run.make_step_inputs(0)
+    run.step(inp, out)
+    torch.cuda.synchronize()
+    ref = ow.expected_decode(w, 1, 0, [0, 1])
+    compare(out[0].cpu().numpy(), ref)
+    assert run.cache.device_status() == 0
