@@ -50,28 +50,61 @@ class Runner:
                                self.w.H, self.w.d, out)
         return out
 
-    def load_prompt(self, compress: bool = True, stream=None):
-        """Append every prompt (layer by layer) and free all prompt spans in one go (Sec. 3.1)."""
+    def load_prompt(self, compress: bool = True, stream=None, mode: str = "compact", block: int = 0):
+        """Append every prompt layer by layer and free the prompt spans (Sec. 3.1).
+
+        mode "compact": append all tokens, then free every span with one compaction ("in one go").
+        mode "free": append with write-time freeing -- spans inside the prompt are never stored.
+        mode "progressive": append `block` tokens per sequence at a time with write-time freeing, and
+        after each block compact the spans that straddled blocks (the paper's for-loop over blocks).
+        """
         w = self.w
-        n_new = self.L.astype(np.int32)
-        kinds = np.concatenate(w.prompt_kinds).astype(np.uint8)
+        if mode == "compact":
+            self._append_tokens(np.zeros(w.b, np.int64), self.L.astype(np.int64), False, stream)
+            if compress:
+                self.compress_prompt(stream)
+            return
+        if mode == "free":
+            self._append_tokens(np.zeros(w.b, np.int64), self.L.astype(np.int64), True, stream)
+            return
+        assert mode == "progressive" and block > 0
+        start = np.zeros(w.b, np.int64)
+        while (start < self.L).any():
+            n = np.minimum(self.L - start, block)
+            self._append_tokens(start, n, True, stream)
+            start = start + n
+            seq, cl, cr = [], [], []
+            for s in range(w.b):
+                for a, c in self.cache.pending_spans(s):
+                    seq.append(s)
+                    cl.append(a)
+                    cr.append(c)
+            if seq:
+                self.cache.compress_spans(seq, cl, cr, stream)
+
+    def _append_tokens(self, start, n, free_closed: bool, stream=None):
+        """Prompt tokens [start[s], start[s] + n[s]) of every sequence, layer by layer."""
+        w = self.w
+        n_new = n.astype(np.int32)
+        kinds = np.concatenate([w.prompt_kinds[s][start[s]:start[s] + n[s]] for s in range(w.b)]).astype(np.uint8)
         N = int(n_new.sum())
-        tok_t = torch.from_numpy(np.concatenate([np.arange(L, dtype=np.int32) for L in self.L])).to(self.device)
-        tok_s = torch.from_numpy(np.repeat(np.arange(w.b, dtype=np.int32), self.L)).to(self.device)
+        if N == 0:
+            return
+        tok_t = torch.from_numpy(np.concatenate([np.arange(start[s], start[s] + n[s], dtype=np.int32)
+                                                 for s in range(w.b)])).to(self.device)
+        tok_s = torch.from_numpy(np.repeat(np.arange(w.b, dtype=np.int32), n)).to(self.device)
         kbuf = torch.empty(N * w.H * w.d, dtype=self.tdt, device=self.device)
         vbuf = torch.empty_like(kbuf)
-        pos = None
+        append = kvc.kvc_append_free_closed if free_closed else kvc.kvc_append
         for m in range(w.M):
             self._fill(synth.K_TENSOR, m, tok_t, tok_s, kbuf, self.kv_scale)
             self._fill(synth.V_TENSOR, m, tok_t, tok_s, vbuf, self.kv_scale)
             if m == 0:
-                pos = self.cache.append(kbuf, vbuf, n_new, kinds, layer=0, stream=stream)
+                pos = self.cache.book.next_positions(n_new, kinds)
+                append(self.cache.handle, 0, kbuf, vbuf, n_new, pos, kinds, stream)
             else:
-                kvc.kvc_append(self.cache.handle, m, kbuf, vbuf, None, None, None, stream)
+                append(self.cache.handle, m, kbuf, vbuf, None, None, None, stream)
         del kbuf, vbuf
-        if compress:
-            self.compress_prompt(stream)
-        return pos
 
     def compress_prompt(self, stream=None):
         seq, cl, cr = [], [], []

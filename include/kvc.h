@@ -88,12 +88,18 @@ void kvc_book_destroy(kvc_book* book);
 /* Tied positions (Sec. 3.1) of tokens about to be appended: n_new[b] tokens per sequence with
  * kinds[sum n_new] (sequence-major); pos_out[sum n_new] continues each sequence's history.
  * A normal token takes the number of normal tokens before it; a sentinel takes the position of
- * the token before it (0 for a sequence's first token).  Validates kinds like kvc_book_append. */
+ * the token before it (0 for a sequence's first token).  Validates kinds like kvc_book_append
+ * (capacity is not checked here). */
 kvc_status kvc_book_next_positions(const kvc_book* book, const int32_t* n_new, const uint8_t* kinds,
                                    int32_t* pos_out);
 
 /* Record n_new[b] tokens per sequence (kinds and positions sequence-major, host). */
 kvc_status kvc_book_append(kvc_book* book, const int32_t* n_new, const uint8_t* kinds, const int32_t* pos);
+
+/* kvc_book_append that frees, as they are recorded, the spans opened and closed among the new
+ * tokens of each sequence (the bookkeeping of kvc_append_free_closed). */
+kvc_status kvc_book_append_free_closed(kvc_book* book, const int32_t* n_new, const uint8_t* kinds,
+                                       const int32_t* pos);
 
 /* Free closed spans: n_spans entries (seq[i], cl[i], cr[i]) given as history indices of the
  * span's <CL> and <CR>.  Each must be a closed span that is not yet freed, listed once. */
@@ -166,6 +172,15 @@ const kvc_book* kvc_get_book(const kvc_cache* cache);
  * its span is freed (paper policy).  Errors: KVC_ERR_CAPACITY, KVC_ERR_SPAN, KVC_ERR_STATE. */
 kvc_status kvc_append(kvc_cache* cache, int layer, const void* k, const void* v, const int32_t* n_new,
                       const int32_t* pos, const uint8_t* kinds, void* stream);
+
+/* kvc_append with write-time freeing (Sec. 3.1: the enclosed KV is freed "in one go" after a
+ * prefix, or block by block for long prefixes): spans that both open and close among the new
+ * tokens of a sequence are freed as the tokens are written -- their <CL> (paper policy) and
+ * enclosed rows are never stored, so no compaction has to move anything for them.  Spans closed
+ * here but opened by an earlier call, or still open, are stored as by kvc_append (free the former
+ * with kvc_compress_spans).  Capacity counts only stored rows.  Same arguments as kvc_append. */
+kvc_status kvc_append_free_closed(kvc_cache* cache, int layer, const void* k, const void* v, const int32_t* n_new,
+                                  const int32_t* pos, const uint8_t* kinds, void* stream);
 
 /* Free closed spans (Sec. 3.1): for each listed (seq, cl, cr) -- history indices of a closed,
  * not yet freed span -- drop its rows (<CL> and the enclosed tokens under the paper policy, only

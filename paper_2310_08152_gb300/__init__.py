@@ -103,6 +103,11 @@ def kvc_book_append(book: int, n_new, kinds, pos):
     _check(lib().kvc_book_append(book, n_new.ctypes.data, kinds.ctypes.data, pos.ctypes.data))
 
 
+def kvc_book_append_free_closed(book: int, n_new, kinds, pos):
+    n_new, kinds, pos = _np(n_new, np.int32), _np(kinds, np.uint8), _np(pos, np.int32)
+    _check(lib().kvc_book_append_free_closed(book, n_new.ctypes.data, kinds.ctypes.data, pos.ctypes.data))
+
+
 def kvc_book_compress(book: int, seq, cl, cr):
     seq, cl, cr = _np(seq, np.int32), _np(cl, np.int64), _np(cr, np.int64)
     _check(lib().kvc_book_compress(book, seq.ctypes.data, cl.ctypes.data, cr.ctypes.data, seq.size))
@@ -163,12 +168,12 @@ class Book:
     def next_positions(self, n_new, kinds):
         return kvc_book_next_positions(self.handle, n_new, kinds)
 
-    def append(self, n_new, kinds, pos=None):
+    def append(self, n_new, kinds, pos=None, free_closed: bool = False):
         if self.readonly:
             raise KvcError(5, "a cache's book is read-only; append through the cache")
         if pos is None:
             pos = self.next_positions(n_new, kinds)
-        kvc_book_append(self.handle, n_new, kinds, pos)
+        (kvc_book_append_free_closed if free_closed else kvc_book_append)(self.handle, n_new, kinds, pos)
         return pos
 
     def compress(self, seq, cl, cr):
@@ -233,6 +238,15 @@ def kvc_append(cache: int, layer: int, k, v, n_new, pos, kinds, stream=None):
     kinds = _np(kinds, np.uint8) if kinds is not None else None
     _check(lib().kvc_append(cache, layer, _ptr(k), _ptr(v), _ptr(n_new), _ptr(pos), _ptr(kinds),
                             _stream_handle(stream)))
+
+
+def kvc_append_free_closed(cache: int, layer: int, k, v, n_new, pos, kinds, stream=None):
+    """kvc_append that frees spans opened and closed among the new tokens as they are written."""
+    n_new = _np(n_new, np.int32) if n_new is not None else None
+    pos = _np(pos, np.int32) if pos is not None else None
+    kinds = _np(kinds, np.uint8) if kinds is not None else None
+    _check(lib().kvc_append_free_closed(cache, layer, _ptr(k), _ptr(v), _ptr(n_new), _ptr(pos), _ptr(kinds),
+                                        _stream_handle(stream)))
 
 
 def kvc_compress_spans(cache: int, seq, cl, cr, stream=None):
@@ -328,8 +342,9 @@ class KVCache:
         base = self.H * int(self.offsets[s]) + h * int(self.capacity[s])
         return plane[base:base + n]
 
-    def append(self, k, v, n_new, kinds, pos=None, layer: int = -1, stream=None):
-        """k, v: device [M or 1][N][H][d] in the cache dtype.  Positions default to the tied positions."""
+    def append(self, k, v, n_new, kinds, pos=None, layer: int = -1, stream=None, free_closed: bool = False):
+        """k, v: device [M or 1][N][H][d] in the cache dtype.  Positions default to the tied positions.
+        free_closed: free spans opened and closed among these tokens as they are written."""
         n_new = _np(n_new, np.int32)
         kinds = _np(kinds, np.uint8)
         if layer <= 0 and pos is None:
@@ -338,7 +353,7 @@ class KVCache:
         nl = self.M if layer < 0 else 1
         _dev(k, "k", self.torch_dtype, nl * N * self.H * self.d)
         _dev(v, "v", self.torch_dtype, nl * N * self.H * self.d)
-        kvc_append(self.handle, layer, k, v, n_new, pos, kinds, stream)
+        (kvc_append_free_closed if free_closed else kvc_append)(self.handle, layer, k, v, n_new, pos, kinds, stream)
         return pos
 
     def compress_spans(self, seq, cl, cr, stream=None):

@@ -40,6 +40,7 @@ SIGNATURES = [
     ("kvc_book_destroy", None, [P]),
     ("kvc_book_next_positions", c_int, [P, P, P, P]),
     ("kvc_book_append", c_int, [P, P, P, P]),
+    ("kvc_book_append_free_closed", c_int, [P, P, P, P]),
     ("kvc_book_compress", c_int, [P, P, P, P, c_int]),
     ("kvc_book_pending_spans", c_int, [P, c_int, P, P, c_int64, P]),
     ("kvc_book_lengths", c_int, [P, P, P]),
@@ -49,6 +50,7 @@ SIGNATURES = [
     ("kvc_destroy", None, [P]),
     ("kvc_get_book", P, [P]),
     ("kvc_append", c_int, [P, c_int, P, P, P, P, P, P]),
+    ("kvc_append_free_closed", c_int, [P, c_int, P, P, P, P, P, P]),
     ("kvc_compress_spans", c_int, [P, P, P, P, c_int, P]),
     ("kvc_decode_attention", c_int, [P, c_int, P, c_float, P, P]),
     ("kvc_decode_attention_static_scratch", c_int, [P, c_int, P, c_float, P, P]),

@@ -13,29 +13,21 @@ Book::Book(int b, Policy policy, const int64_t* capacity) : b_(b), policy_(polic
   }
 }
 
-bool Book::check_append(const int32_t* n_new, const uint8_t* kinds, std::string& err, int& code) const {
+bool Book::check_append(const int32_t* n_new, const uint8_t* kinds, std::string& err, int& code,
+                        bool free_in_block, bool check_capacity) const {
   int64_t off = 0;
   char buf[256];
   for (int s = 0; s < b_; ++s) {
-    const Seq& q = seqs_[s];
     if (n_new[s] < 0) {
       std::snprintf(buf, sizeof buf, "n_new[%d] = %d is negative", s, n_new[s]);
       err = buf;
       code = 1;
       return false;
     }
-    if (q.stored + n_new[s] > q.cap) {
-      std::snprintf(buf, sizeof buf, "sequence %d: %lld stored + %d new rows exceed capacity %lld", s,
-                    (long long)q.stored, n_new[s], (long long)q.cap);
-      err = buf;
-      code = 3;
-      return false;
-    }
-    if (q.kind.size() + (size_t)n_new[s] >= (size_t)INT32_MAX) {
-      err = "history index would overflow int32";
-      code = 3;
-      return false;
-    }
+  }
+  // kinds first (the kept count below relies on well-formed spans), then capacity
+  for (int s = 0; s < b_; ++s) {
+    const Seq& q = seqs_[s];
     bool open = q.open;
     for (int t = 0; t < n_new[s]; ++t) {
       uint8_t k = kinds[off + t];
@@ -66,7 +58,55 @@ bool Book::check_append(const int32_t* n_new, const uint8_t* kinds, std::string&
     }
     off += n_new[s];
   }
+  if (!check_capacity) return true;
+  std::vector<uint8_t> kept;
+  if (free_in_block) kept_in_block(n_new, kinds, kept);
+  off = 0;
+  for (int s = 0; s < b_; ++s) {
+    const Seq& q = seqs_[s];
+    int64_t stored_new = n_new[s];
+    if (free_in_block) {
+      stored_new = 0;
+      for (int t = 0; t < n_new[s]; ++t) stored_new += kept[off + t];
+    }
+    if (q.stored + stored_new > q.cap) {
+      std::snprintf(buf, sizeof buf, "sequence %d: %lld stored + %lld new rows exceed capacity %lld", s,
+                    (long long)q.stored, (long long)stored_new, (long long)q.cap);
+      err = buf;
+      code = 3;
+      return false;
+    }
+    if (q.kind.size() + (size_t)n_new[s] >= (size_t)INT32_MAX) {
+      err = "history index would overflow int32";
+      code = 3;
+      return false;
+    }
+    off += n_new[s];
+  }
   return true;
+}
+
+void Book::kept_in_block(const int32_t* n_new, const uint8_t* kinds, std::vector<uint8_t>& kept) const {
+  int64_t total = 0;
+  for (int s = 0; s < b_; ++s) total += n_new[s];
+  kept.assign((size_t)total, 1);
+  int64_t off = 0;
+  for (int s = 0; s < b_; ++s) {
+    int64_t open_at = -1;  // index (within this call) of a <CL> opened by these tokens
+    for (int t = 0; t < n_new[s]; ++t) {
+      const uint8_t k = kinds[off + t];
+      if (k == CL) {
+        open_at = t;
+      } else if (k == CR && open_at >= 0) {  // opened and closed here: free <CL> (paper) and the interior
+        const int64_t lo = policy_ == POLICY_PAPER ? open_at : open_at + 1;
+        for (int64_t u = lo; u < t; ++u) kept[off + u] = 0;
+        open_at = -1;
+      } else if (k == CR) {
+        open_at = -1;  // closes a span opened before this call: stored, freed later by compaction
+      }
+    }
+    off += n_new[s];
+  }
 }
 
 void Book::next_positions(const int32_t* n_new, const uint8_t* kinds, int32_t* pos_out) const {
@@ -92,15 +132,19 @@ void Book::next_positions(const int32_t* n_new, const uint8_t* kinds, int32_t* p
   }
 }
 
-void Book::apply_append(const int32_t* n_new, const uint8_t* kinds, const int32_t* pos) {
+void Book::apply_append(const int32_t* n_new, const uint8_t* kinds, const int32_t* pos, const uint8_t* kept) {
   int64_t off = 0;
   for (int s = 0; s < b_; ++s) {
     Seq& q = seqs_[s];
+    const int64_t T0 = (int64_t)q.kind.size();
+    int64_t stored_new = 0;
+    bool freed_any = false;
     for (int t = 0; t < n_new[s]; ++t) {
       uint8_t k = kinds[off + t];
       int64_t j = (int64_t)q.kind.size();
       q.kind.push_back(k);
       q.pos.push_back(pos[off + t]);
+      stored_new += kept ? kept[off + t] : 1;
       if (k == NORMAL) {
         q.normals += 1;
       } else if (k == CL) {
@@ -109,11 +153,19 @@ void Book::apply_append(const int32_t* n_new, const uint8_t* kinds, const int32_
         q.spans.push_back(sp);
         q.open = true;
       } else {
-        q.spans.back().cr = j;
+        Span& sp = q.spans.back();
+        sp.cr = j;
         q.open = false;
+        if (kept && sp.cl >= T0) {  // opened and closed in this call: freed as it was written
+          sp.freed = true;
+          const int64_t lo = policy_ == POLICY_PAPER ? sp.cl : sp.cl + 1;
+          if (lo < sp.cr) q.freed.emplace_back(lo, sp.cr);
+          freed_any = true;
+        }
       }
     }
-    q.stored += n_new[s];
+    if (freed_any) rebuild_prefix(q);
+    q.stored += stored_new;
     off += n_new[s];
   }
 }

@@ -52,10 +52,16 @@ class Book {
   int64_t stored(int s) const { return seqs_[s].stored; }
   int64_t history(int s) const { return (int64_t)seqs_[s].kind.size(); }
 
-  // Validation only (no state change).  On error returns false and sets `err`.
-  bool check_append(const int32_t* n_new, const uint8_t* kinds, std::string& err, int& code) const;
+  // Validation only (no state change).  On error returns false and sets `err`.  With
+  // free_in_block, the capacity check counts only the rows that will be stored.
+  bool check_append(const int32_t* n_new, const uint8_t* kinds, std::string& err, int& code,
+                    bool free_in_block = false, bool check_capacity = true) const;
   void next_positions(const int32_t* n_new, const uint8_t* kinds, int32_t* pos_out) const;
-  void apply_append(const int32_t* n_new, const uint8_t* kinds, const int32_t* pos);
+  // Which of the new tokens are stored when spans opened and closed among them are freed as they
+  // are written (their <CL> under the paper policy, and the enclosed tokens, are never stored).
+  void kept_in_block(const int32_t* n_new, const uint8_t* kinds, std::vector<uint8_t>& kept) const;
+  // kept == nullptr: every new token is stored.
+  void apply_append(const int32_t* n_new, const uint8_t* kinds, const int32_t* pos, const uint8_t* kept = nullptr);
 
   bool plan_compress(const int32_t* seq, const int64_t* cl, const int64_t* cr, int n, std::vector<CompactSeq>& plan,
                      std::string& err) const;

@@ -119,8 +119,8 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
 // [n_copy, n_copy + n_rot) rotate one pair of 8-column vectors of K for every head of one token.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) append_kernel(Geometry g, Static st, Buffers buf,
-                                                     const TokPlan* __restrict__ plan, int64_t ntok, int m0,
-                                                     int n_layers, int write_meta,
+                                                     const TokPlan* __restrict__ plan, int64_t ntok, int64_t n_in,
+                                                     int m0, int n_layers, int write_meta,
                                                      const uint16_t* __restrict__ k_in,
                                                      const uint16_t* __restrict__ v_in) {
   constexpr int VPR = D / 8;
@@ -143,7 +143,7 @@ __global__ void __launch_bounds__(256) append_kernel(Geometry g, Static st, Buff
       const TokPlan tp = plan[tok];
       const bool is_v = c < VPR;
       const int vec = is_v ? c : 2 * hv + (c - VPR);
-      const uint16_t* src = (is_v ? v_in : k_in) + (((int64_t)l * ntok + tok) * H + h) * D;
+      const uint16_t* src = (is_v ? v_in : k_in) + (((int64_t)l * n_in + tp.in_tok) * H + h) * D;
       uint16_t* dst = (is_v ? buf.v : buf.k) +
                       ((int64_t)(m0 + l) * plane + st.seq_row0[tp.s] + (int64_t)h * st.cap[tp.s] + tp.row) * D;
       *reinterpret_cast<uint4*>(dst + vec * 8) = __ldg(reinterpret_cast<const uint4*>(src + vec * 8));
@@ -162,7 +162,7 @@ __global__ void __launch_bounds__(256) append_kernel(Geometry g, Static st, Buff
 #pragma unroll
       for (int e = 0; e < 8; ++e) rope_sincos(tp.pos, st.rope_g[vec * 8 + e], &sn[e], &cs[e]);
       for (int h = 0; h < H; ++h) {
-        const uint16_t* src = k_in + (((int64_t)l * ntok + tok) * H + h) * D;
+        const uint16_t* src = k_in + (((int64_t)l * n_in + tp.in_tok) * H + h) * D;
         uint16_t* dst =
             buf.k + ((int64_t)(m0 + l) * plane + st.seq_row0[tp.s] + (int64_t)h * st.cap[tp.s] + tp.row) * D;
         uint4 a = __ldg(reinterpret_cast<const uint4*>(src + vec * 8));
@@ -907,7 +907,7 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
 
 template <typename T, int D>
 cudaError_t launch_append_t(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t ntok,
-                            int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
+                            int64_t n_in, int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
                             cudaStream_t stream) {
   constexpr int VPR = D / 8;
   const int hv = g.rot / 16;
@@ -916,7 +916,7 @@ cudaError_t launch_append_t(const Geometry& g, const Static& st, const Buffers& 
   int64_t blocks = (n_items + 255) / 256;
   if (blocks > 65535LL * 16) blocks = 65535LL * 16;
   if (blocks < 1) blocks = 1;
-  append_kernel<T, D><<<(unsigned)blocks, 256, 0, stream>>>(g, st, buf, plan, ntok, m0, n_layers, write_meta ? 1 : 0,
+  append_kernel<T, D><<<(unsigned)blocks, 256, 0, stream>>>(g, st, buf, plan, ntok, n_in, m0, n_layers, write_meta ? 1 : 0,
                                                             static_cast<const uint16_t*>(k_in),
                                                             static_cast<const uint16_t*>(v_in));
   return cudaGetLastError();
@@ -942,13 +942,14 @@ cudaError_t by_dhead(int D, F&& f) {
 
 bool dhead_supported(int D) { return D == 64 || D == 80 || D == 96 || D == 128; }
 
-cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t ntok,
-                          int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
+cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t n_plan,
+                          int64_t n_in, int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
                           cudaStream_t stream) {
   return by_dhead(g.D, [&](auto dc) {
     constexpr int D = decltype(dc)::value;
-    if (g.dtype == 1) return launch_append_t<BF16T, D>(g, st, buf, plan, ntok, m0, n_layers, write_meta, k_in, v_in, stream);
-    return launch_append_t<F16T, D>(g, st, buf, plan, ntok, m0, n_layers, write_meta, k_in, v_in, stream);
+    if (g.dtype == 1)
+      return launch_append_t<BF16T, D>(g, st, buf, plan, n_plan, n_in, m0, n_layers, write_meta, k_in, v_in, stream);
+    return launch_append_t<F16T, D>(g, st, buf, plan, n_plan, n_in, m0, n_layers, write_meta, k_in, v_in, stream);
   });
 }
 

@@ -13,9 +13,10 @@ struct DState {
   int32_t len, begin, mask_lo, mask_hi, qpos, pad0, pad1, pad2;
 };
 
-// One appended token: its sequence, destination row, position and history index.
+// One stored token: its sequence, destination row, position, history index, and its index among
+// the input tokens of the call (tokens freed as they are written have no plan entry).
 struct TokPlan {
-  int32_t s, row, pos, orig;
+  int32_t s, row, pos, orig, in_tok, pad0, pad1, pad2;
 };
 
 // One sequence of a compaction; its drop ranges (history indices, [lo, hi)) are
@@ -54,8 +55,9 @@ constexpr int kMaxDecodeWorkers = 8192;
 
 bool dhead_supported(int D);
 
-cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t ntok,
-                          int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
+// Writes the n_plan stored tokens of a call whose inputs hold n_in tokens per layer.
+cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t n_plan,
+                          int64_t n_in, int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
                           cudaStream_t stream);
 
 cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& buf, const AffSeq* aff, int n_aff,

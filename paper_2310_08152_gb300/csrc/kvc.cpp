@@ -201,7 +201,8 @@ struct kvc_cache {
   PinnedRing ring;
   // token batch in progress: layers [0, layers_done) written
   int layers_done = 0;
-  int64_t batch_ntok = 0;
+  int64_t batch_ntok = 0;  // stored tokens of the batch (plan entries)
+  int64_t batch_nin = 0;   // input tokens of the batch (per layer of k, v)
   // decode readiness of the uploaded state
   bool decode_ok = false;
   std::string decode_err;
@@ -397,8 +398,13 @@ static kvc_status book_check_append(const kvc::Book& B, const int32_t* n_new, co
 kvc_status kvc_book_next_positions(const kvc_book* book, const int32_t* n_new, const uint8_t* kinds,
                                    int32_t* pos_out) {
   if (!book) return fail(KVC_ERR_INVALID_ARG, "book is NULL");
-  kvc_status st = book_check_append(book->book, n_new, kinds);
-  if (st != KVC_OK) return st;
+  if (!n_new) return fail(KVC_ERR_INVALID_ARG, "n_new is NULL");
+  int64_t N = 0;
+  for (int s = 0; s < book->book.b(); ++s) N += n_new[s] > 0 ? n_new[s] : 0;
+  if (N > 0 && !kinds) return fail(KVC_ERR_INVALID_ARG, "kinds is NULL");
+  std::string err;
+  int code = 0;  // positions need well-formed kinds, not capacity
+  if (!book->book.check_append(n_new, kinds, err, code, false, false)) return fail((kvc_status)code, "%s", err.c_str());
   if (!pos_out) return fail(KVC_ERR_INVALID_ARG, "pos_out is NULL");
   book->book.next_positions(n_new, kinds, pos_out);
   return ok();
@@ -410,6 +416,22 @@ kvc_status kvc_book_append(kvc_book* book, const int32_t* n_new, const uint8_t* 
   if (st != KVC_OK) return st;
   if (!pos) return fail(KVC_ERR_INVALID_ARG, "pos is NULL");
   book->book.apply_append(n_new, kinds, pos);
+  return ok();
+}
+
+kvc_status kvc_book_append_free_closed(kvc_book* book, const int32_t* n_new, const uint8_t* kinds,
+                                       const int32_t* pos) {
+  if (!book) return fail(KVC_ERR_INVALID_ARG, "book is NULL");
+  if (!n_new) return fail(KVC_ERR_INVALID_ARG, "n_new is NULL");
+  int64_t N = 0;
+  for (int s = 0; s < book->book.b(); ++s) N += n_new[s] > 0 ? n_new[s] : 0;
+  if (N > 0 && (!kinds || !pos)) return fail(KVC_ERR_INVALID_ARG, "kinds/pos are NULL");
+  std::string err;
+  int code = 0;
+  if (!book->book.check_append(n_new, kinds, err, code, true)) return fail((kvc_status)code, "%s", err.c_str());
+  std::vector<uint8_t> kept;
+  book->book.kept_in_block(n_new, kinds, kept);
+  book->book.apply_append(n_new, kinds, pos, kept.data());
   return ok();
 }
 
@@ -511,8 +533,8 @@ void kvc_destroy(kvc_cache* cache) { delete cache; }
 
 const kvc_book* kvc_get_book(const kvc_cache* cache) { return cache ? &cache->bk : nullptr; }
 
-kvc_status kvc_append(kvc_cache* c, int layer, const void* k, const void* v, const int32_t* n_new, const int32_t* pos,
-                      const uint8_t* kinds, void* stream_) {
+static kvc_status append_impl(kvc_cache* c, int layer, const void* k, const void* v, const int32_t* n_new,
+                              const int32_t* pos, const uint8_t* kinds, void* stream_, bool free_in_block) {
   if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
   const int M = c->cfg.M;
@@ -522,10 +544,14 @@ kvc_status kvc_append(kvc_cache* c, int layer, const void* k, const void* v, con
   if (starts) {
     if (c->layers_done != M)
       return fail(KVC_ERR_STATE, "layers %d..%d of the previous tokens are not written yet", c->layers_done, M - 1);
-    kvc_status st = book_check_append(c->bk.book, n_new, kinds);
-    if (st != KVC_OK) return st;
+    if (!n_new) return fail(KVC_ERR_INVALID_ARG, "n_new is NULL");
     int64_t N = 0;
-    for (int s = 0; s < c->cfg.b; ++s) N += n_new[s];
+    for (int s = 0; s < c->cfg.b; ++s) N += n_new[s] > 0 ? n_new[s] : 0;
+    if (N > 0 && !kinds) return fail(KVC_ERR_INVALID_ARG, "kinds is NULL");
+    std::string err;
+    int code = 0;
+    if (!c->bk.book.check_append(n_new, kinds, err, code, free_in_block))
+      return fail((kvc_status)code, "%s", err.c_str());
     if (N > 0 && !pos) return fail(KVC_ERR_INVALID_ARG, "pos is NULL");
   } else if (c->layers_done != layer) {
     return fail(KVC_ERR_STATE, "layer %d appended out of order (expected %d)", layer, c->layers_done);
@@ -536,44 +562,65 @@ kvc_status kvc_append(kvc_cache* c, int layer, const void* k, const void* v, con
   if (starts) {
     int64_t N = 0;
     for (int s = 0; s < c->cfg.b; ++s) N += n_new[s];
+    std::vector<uint8_t> kept;
+    if (free_in_block) c->bk.book.kept_in_block(n_new, kinds, kept);
+    int64_t n_plan = 0;
+    for (int64_t t = 0; t < N; ++t) n_plan += free_in_block ? kept[t] : 1;
     // destination rows before the book moves on
     std::vector<int64_t> row0(c->cfg.b), orig0(c->cfg.b);
     for (int s = 0; s < c->cfg.b; ++s) {
       row0[s] = c->bk.book.stored(s);
       orig0[s] = c->bk.book.history(s);
     }
-    const size_t bytes = c->ws.dyn_payload + sizeof(kvc::TokPlan) * (size_t)N;
+    const size_t bytes = c->ws.dyn_payload + sizeof(kvc::TokPlan) * (size_t)n_plan;
     cudaError_t e;
     unsigned char* img = c->ring.reserve(bytes, &e);
     if (!img) return cuda_fail(e, "staging");
-    c->bk.book.apply_append(n_new, kinds, pos);
+    c->bk.book.apply_append(n_new, kinds, pos, free_in_block ? kept.data() : nullptr);
     c->fill_state(img);
     kvc::TokPlan* tp = reinterpret_cast<kvc::TokPlan*>(img + c->ws.dyn_payload);
-    int64_t t = 0;
+    int64_t t = 0, w = 0;
     for (int s = 0; s < c->cfg.b; ++s) {
+      int64_t row = row0[s];
       for (int i = 0; i < n_new[s]; ++i, ++t) {
-        tp[t].s = s;
-        tp[t].row = (int32_t)(row0[s] + i);
-        tp[t].pos = pos[t];
-        tp[t].orig = (int32_t)(orig0[s] + i);
+        if (free_in_block && !kept[t]) continue;  // freed as it is written: never stored
+        tp[w].s = s;
+        tp[w].row = (int32_t)row++;
+        tp[w].pos = pos[t];
+        tp[w].orig = (int32_t)(orig0[s] + i);
+        tp[w].in_tok = (int32_t)t;
+        tp[w].pad0 = tp[w].pad1 = tp[w].pad2 = 0;
+        ++w;
       }
     }
     e = c->ring.commit(c->wsp(c->ws.dyn), bytes, stream);
     if (e != cudaSuccess) return cuda_fail(e, "upload append plan");
-    c->batch_ntok = N;
+    c->batch_ntok = n_plan;
+    c->batch_nin = N;
     c->layers_done = 0;
   }
   const int m0 = layer < 0 ? 0 : layer;
   const int nl = layer < 0 ? M : 1;
   if (c->batch_ntok > 0) {
     const kvc::TokPlan* plan = reinterpret_cast<const kvc::TokPlan*>(c->wsp(c->ws.dyn + c->ws.dyn_payload));
-    cudaError_t e = kvc::launch_append(g, c->stat(), c->bufs(), plan, c->batch_ntok, m0, nl, m0 == 0, k, v, stream);
+    cudaError_t e = kvc::launch_append(g, c->stat(), c->bufs(), plan, c->batch_ntok, c->batch_nin, m0, nl, m0 == 0, k,
+                                       v, stream);
     if (e != cudaSuccess) return cuda_fail(e, "append kernel");
     c->launches += 1;
     c->last_was_decode = false;
   }
   c->layers_done = m0 + nl;
   return ok();
+}
+
+kvc_status kvc_append(kvc_cache* c, int layer, const void* k, const void* v, const int32_t* n_new, const int32_t* pos,
+                      const uint8_t* kinds, void* stream) {
+  return append_impl(c, layer, k, v, n_new, pos, kinds, stream, false);
+}
+
+kvc_status kvc_append_free_closed(kvc_cache* c, int layer, const void* k, const void* v, const int32_t* n_new,
+                                  const int32_t* pos, const uint8_t* kinds, void* stream) {
+  return append_impl(c, layer, k, v, n_new, pos, kinds, stream, true);
 }
 
 kvc_status kvc_compress_spans(kvc_cache* c, const int32_t* seq, const int64_t* cl, const int64_t* cr, int n_spans,

@@ -243,3 +243,55 @@ def test_cache_fails_loudly_without_a_gpu():
         assert rc == 6  # KVC_ERR_CUDA: no silent CPU path
     finally:
         kvc.kvc_destroy(h)
+
+
+@pytest.mark.parametrize("policy", [kvc.POLICY_PAPER, kvc.POLICY_KEEP_CL])
+def test_book_write_time_freeing_matches_oracle(policy):
+    """Spans opened and closed within one append are freed as they are written (Sec. 3.1, freeing in
+    one go / block by block); the stored rows equal the oracle's rows left after freeing them, and a
+    later compaction of the spans that straddled calls gives the same rows as freeing everything."""
+    rng = np.random.default_rng(21)
+    b = 3
+    book = kvc.Book(b, np.full(b, 5000, np.int64), policy)
+    hist = [np.zeros(0, np.uint8) for _ in range(b)]
+    freed = [[] for _ in range(b)]
+    open_ = [False] * b
+    for rnd in range(30):
+        n_new = rng.integers(0, 40, size=b).astype(np.int32)
+        parts = []
+        for s in range(b):
+            k, open_[s] = _random_kinds(rng, int(n_new[s]), open_[s])
+            parts.append(k)
+        book.append(n_new, np.concatenate(parts), free_closed=True)
+        for s in range(b):
+            T0 = hist[s].size
+            hist[s] = np.concatenate([hist[s], parts[s]])
+            closed, _ = orc.pair_spans(hist[s])
+            freed[s] += [(a, c) for a, c in closed if a >= T0]  # opened and closed in this call
+        ln, _ = book.lengths()
+        for s in range(b):
+            rows = orc.stored_rows(hist[s].size, freed[s], policy)
+            assert np.array_equal(book.layout(s)["stored_orig"], rows)
+            assert ln[s] == rows.size
+            closed, _ = orc.pair_spans(hist[s])
+            assert book.pending_spans(s) == [sp for sp in closed if sp not in freed[s]]
+    # free what straddled calls: the same rows as freeing every closed span
+    seq, cl, cr = [], [], []
+    for s in range(b):
+        for a, c in book.pending_spans(s):
+            seq.append(s)
+            cl.append(a)
+            cr.append(c)
+    if seq:
+        book.compress(seq, cl, cr)
+    for s in range(b):
+        closed, _ = orc.pair_spans(hist[s])
+        assert np.array_equal(book.layout(s)["stored_orig"], orc.stored_rows(hist[s].size, closed, policy))
+
+
+def test_write_time_freeing_capacity_counts_stored_rows():
+    book = kvc.Book(1, [5])
+    # 9 tokens, of which <CL> and 4 enclosed are freed at write time: 4 stored rows fit capacity 5
+    book.append([9], [NORMAL, CL, NORMAL, NORMAL, NORMAL, NORMAL, CR, NORMAL, NORMAL], free_closed=True)
+    assert book.lengths()[0][0] == 4
+    assert _err(book.append, [2], [NORMAL, NORMAL]) == 3

@@ -241,3 +241,23 @@ def test_bounded_wait_reports_timeout_and_context_survives():
     ref = ow.expected_decode(w, 1, 0, [0, 1])
     compare(out[0].cpu().numpy(), ref)
     assert run.cache.device_status() == 0
+
+
+@pytest.mark.parametrize("mode,block", [("free", 0), ("progressive", 100), ("progressive", 64)])
+def test_write_time_freeing_prompt_modes(mode, block):
+    # freeing at write time (in one go, or block by block with compaction of the spans that straddle
+    # blocks) leaves exactly the rows the paper keeps; decode over them matches the oracle
+    for w in (wl.opt13b(b=3, L=640, M=2), wl.ragged(b=5, lmin=64, lmax=700, M=2, steps=4)):
+        run = harness.Runner(w, steps=3)
+        run.load_prompt(mode=mode, block=block)
+        check_metadata(run, 0)
+        for s in range(w.b):
+            check_rows(run, 0, 1, s, [0, 17])
+        out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device="cuda")
+        for g in range(3):
+            inp = run.make_step_inputs(g)
+            run.step(inp, out)
+            torch.cuda.synchronize()
+            for m in range(w.M):
+                compare(out[m].cpu().numpy(), ow.expected_decode(w, g + 1, m, list(range(w.b))), f"{mode} {g} {m}")
+        assert run.cache.device_status() == 0
