@@ -335,6 +335,25 @@ def time_prompt_compaction(run, w):
             "frac": (gbs / peak) if gbs else None, "peak_kind": kind}
 
 
+def time_prompt_write_time_freeing(w, steps_total, dev):
+    """The same prompts ingested with write-time freeing (spans never stored, nothing to compact):
+    the append calls' time, against append + compaction of the one-go path."""
+    import torch
+
+    import harness
+
+    run = harness.Runner(w, steps_total, device=dev)
+    ev = []
+    run.load_prompt(mode="free", timer=ev)
+    torch.cuda.synchronize()
+    ms = sum(a.elapsed_time(b) for a, b in ev)
+    stored = int(run.cache.lengths()[0].sum())
+    del run
+    torch.cuda.empty_cache()
+    return {"mode": "write-time freeing (kvc_append_free_closed)", "append_ms": ms,
+            "rows_written_per_stream": stored, "rows_in_prompt_per_stream": int(w.prompt_len.sum())}
+
+
 def run_kvc(args, w):
     import torch
     import torch.distributed as dist
@@ -351,8 +370,12 @@ def run_kvc(args, w):
 
     # ---------------- device-resident run ----------------
     run = harness.Runner(w, steps_total, device=dev)
-    run.load_prompt(compress=False)
+    append_ev = []
+    run.load_prompt(compress=False, timer=append_ev)
     compaction = time_prompt_compaction(run, w)
+    torch.cuda.synchronize()
+    compaction["prompt_append_ms"] = sum(a.elapsed_time(b) for a, b in append_ev)
+    prompt_free = time_prompt_write_time_freeing(w, steps_total, dev)
     inputs = [run.make_step_inputs(g) for g in range(steps_total)]
     out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device=dev)
     torch.cuda.synchronize()
@@ -434,6 +457,7 @@ def run_kvc(args, w):
                             "tile_rows": plan["tile_rows"], "stages": plan["stages"]},
             "decode_share_of_step": dec_total_s / elapsed,
             "compaction": compaction,
+            "prompt_write_time_freeing": prompt_free,
             "gpu_launches": launches,
             "device_status": status,
             "clocks": clk,

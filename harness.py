@@ -50,7 +50,7 @@ class Runner:
                                self.w.H, self.w.d, out)
         return out
 
-    def load_prompt(self, compress: bool = True, stream=None, mode: str = "compact", block: int = 0):
+    def load_prompt(self, compress: bool = True, stream=None, mode: str = "compact", block: int = 0, timer=None):
         """Append every prompt layer by layer and free the prompt spans (Sec. 3.1).
 
         mode "compact": append all tokens, then free every span with one compaction ("in one go").
@@ -60,18 +60,18 @@ class Runner:
         """
         w = self.w
         if mode == "compact":
-            self._append_tokens(np.zeros(w.b, np.int64), self.L.astype(np.int64), False, stream)
+            self._append_tokens(np.zeros(w.b, np.int64), self.L.astype(np.int64), False, stream, timer)
             if compress:
                 self.compress_prompt(stream)
             return
         if mode == "free":
-            self._append_tokens(np.zeros(w.b, np.int64), self.L.astype(np.int64), True, stream)
+            self._append_tokens(np.zeros(w.b, np.int64), self.L.astype(np.int64), True, stream, timer)
             return
         assert mode == "progressive" and block > 0
         start = np.zeros(w.b, np.int64)
         while (start < self.L).any():
             n = np.minimum(self.L - start, block)
-            self._append_tokens(start, n, True, stream)
+            self._append_tokens(start, n, True, stream, timer)
             start = start + n
             seq, cl, cr = [], [], []
             for s in range(w.b):
@@ -82,8 +82,9 @@ class Runner:
             if seq:
                 self.cache.compress_spans(seq, cl, cr, stream)
 
-    def _append_tokens(self, start, n, free_closed: bool, stream=None):
-        """Prompt tokens [start[s], start[s] + n[s]) of every sequence, layer by layer."""
+    def _append_tokens(self, start, n, free_closed: bool, stream=None, timer=None):
+        """Prompt tokens [start[s], start[s] + n[s]) of every sequence, layer by layer.  timer: a list
+        that receives a (start, end) CUDA event pair around every append call."""
         w = self.w
         n_new = n.astype(np.int32)
         kinds = np.concatenate([w.prompt_kinds[s][start[s]:start[s] + n[s]] for s in range(w.b)]).astype(np.uint8)
@@ -99,11 +100,17 @@ class Runner:
         for m in range(w.M):
             self._fill(synth.K_TENSOR, m, tok_t, tok_s, kbuf, self.kv_scale)
             self._fill(synth.V_TENSOR, m, tok_t, tok_s, vbuf, self.kv_scale)
+            if timer is not None:
+                ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                ev[0].record(stream)
             if m == 0:
                 pos = self.cache.book.next_positions(n_new, kinds)
                 append(self.cache.handle, 0, kbuf, vbuf, n_new, pos, kinds, stream)
             else:
                 append(self.cache.handle, m, kbuf, vbuf, None, None, None, stream)
+            if timer is not None:
+                ev[1].record(stream)
+                timer.append(ev)
         del kbuf, vbuf
 
     def compress_prompt(self, stream=None):
