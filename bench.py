@@ -44,6 +44,10 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="budget of the CPU-baseline sample")
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (small profiling runs)")
+    ap.add_argument("--capacity-sweep", action="store_true",
+                    help="largest batch under a KV-memory cap per compression ratio, and its throughput")
+    ap.add_argument("--caps", default="12,24,180", help="KV-memory caps in GB for --capacity-sweep")
+    ap.add_argument("--ratios", default="0,0.5,0.8,0.9", help="compression ratios for --capacity-sweep")
     return ap.parse_args()
 
 
@@ -354,6 +358,55 @@ def time_prompt_write_time_freeing(w, steps_total, dev):
             "rows_written_per_stream": stored, "rows_in_prompt_per_stream": int(w.prompt_len.sum())}
 
 
+def run_capacity_sweep(args):
+    """Largest batch whose compressed KV cache fits a memory cap, and its decode-step throughput, for
+    several compression ratios: a synthetic restatement of the paper's throughput-vs-VRAM experiment
+    (Sec. 4.3, Fig. 2 bottom right) and memory experiment (App. C, Fig. 4).  The cap covers the KV
+    cache only (no model weights: this path has none).  Prompts are ingested with write-time freeing,
+    so a sequence holds only its kept rows plus the generated ones."""
+    import torch
+
+    import harness
+    import paper_2310_08152_gb300 as kvc
+    from synth import workloads as wl
+
+    torch.cuda.set_device(0)
+    caps_gb = [float(x) for x in args.caps.split(",")]
+    ratios = [float(x) for x in args.ratios.split(",")]
+    steps = args.steps
+    for cap_gb in caps_gb:
+        for r in ratios:
+            probe = wl.throughput_3b(r, b=1, steps=steps)
+            kept = int(probe.prompt_len[0]) - sum(c - a for a, c in probe.prompt_spans[0])  # paper policy
+            per_seq = probe.M * 2 * probe.H * probe.d * 2 * (kept + args.warmup + steps)
+            b = int(cap_gb * 1e9 // per_seq)
+            b = max(1, min(b, 4096))
+            w = wl.throughput_3b(r, b=b, steps=steps)
+            # capacity: only what a sequence stores (kept prompt rows + generated rows)
+            run = harness.Runner(w, args.warmup + steps, capacity=np.full(b, kept + args.warmup + steps))
+            run.load_prompt(mode="free")
+            # every generated token is a normal token: one step's inputs serve every step (the values
+            # read from the cache, not these, set the work)
+            inp = run.make_step_inputs(0)
+            out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device="cuda")
+            for g in range(args.warmup):
+                run.step(inp, out)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for g in range(args.warmup, args.warmup + steps):
+                run.step(inp, out)
+            e1.record()
+            torch.cuda.synchronize()
+            sec = e0.elapsed_time(e1) / 1e3
+            kv_gb = run.cache.sizes["k"] * 2 / 1e9
+            print(json.dumps({"sweep": "capacity", "kv_cap_gb": cap_gb, "ratio": r, "batch": b,
+                              "kept_prompt_rows": kept, "kv_allocated_gb": kv_gb, "tokens_per_s": w.b * steps / sec,
+                              "ms_per_step": sec / steps * 1e3, "status": run.cache.device_status()}), flush=True)
+            del run, inp, out
+            torch.cuda.empty_cache()
+
+
 def run_kvc(args, w):
     import torch
     import torch.distributed as dist
@@ -524,6 +577,9 @@ def main():
     args = parse()
     from synth import workloads as wl
 
+    if args.capacity_sweep:
+        run_capacity_sweep(args)
+        return
     w = wl.by_name(args.workload)
     if args.layers:
         import dataclasses

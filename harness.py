@@ -29,13 +29,13 @@ class StepInputs:
 
 class Runner:
     def __init__(self, w: wl.Workload, steps: int, policy: int = kvc.POLICY_PAPER, device=None,
-                 capacity_slack: int = 0):
+                 capacity_slack: int = 0, capacity=None):
         self.w = w
         self.steps = steps
         self.policy = policy
         self.device = torch.device("cuda", 0) if device is None else torch.device(device)
         self.tdt = torch.float16 if w.dtype == "f16" else torch.bfloat16
-        cap = w.capacity(steps) + capacity_slack
+        cap = (w.capacity(steps) if capacity is None else np.asarray(capacity, np.int64)) + capacity_slack
         self.cache = kvc.KVCache(w.M, w.H, w.d, cap, w.dtype, w.rotary_dim, w.rope_base, policy, device=self.device)
         self.L = w.prompt_len.copy()
         self.open_cl = [-1] * w.b      # history index of an open <CL>

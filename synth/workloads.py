@@ -214,6 +214,23 @@ def ragged(b: int = 128, lmin: int = 256, lmax: int = 8192, M: int = 24, steps: 
                     extra={"opens": opens, "gaps": gaps})
 
 
+def throughput_3b(ratio: float, b: int, prefix: int = 800, M: int = 32, steps: int = 64) -> Workload:
+    """The paper's throughput setting (Sec. 4.3): RedPajama-3B shapes (M=32, H=32, d=80, fp16, RoPE),
+    a dummy prefix of 800 tokens transformed to compression ratio r, then normal generated tokens.
+    Spans: one <CL>..<CR> pair per 64-token block, <CL> first, round(64 r) enclosed tokens."""
+    interior = int(round(64 * ratio))
+    if interior == 0:
+        kinds, spans = np.zeros(prefix, dtype=np.uint8), []
+    else:
+        assert interior + 2 <= 64, "r too high for one span per 64-token block"
+        kinds, spans = block_kinds(prefix, interior, cl_off=0)
+    return Workload(f"throughput3b_r{ratio:.2f}", 3, M=M, H=32, d=80, dtype="f16", b=b,
+                    prompt_kinds=[kinds.copy() for _ in range(b)], prompt_spans=[list(spans) for _ in range(b)],
+                    n_steps=steps, gen_kind=_normal_gen, scale=1.0 / math.sqrt(80), rotary_dim=80,
+                    rope_base=10000.0, seed=SEED_BASE + 5,
+                    note=f"3B rotary shapes, prefix {prefix} at r={ratio:.2f} ({interior} enclosed per 64), b={b}")
+
+
 def by_name(name: str, **kw) -> Workload:
     table = {"tiny": tiny, "opt1.3b": opt13b, "opt1.3b_r0": opt13b_uncompressed, "opt2.7b": opt27b,
              "ragged": ragged}
