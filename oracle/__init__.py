@@ -53,6 +53,8 @@ def lib():
         L.orc_attend.argtypes = [i32, i32, p, p, p, p, p, i64, f64, i32, f64, i32, p]
         L.orc_masked_decode.argtypes = [i64, i64, i32, i32, p, p, p, p, p, p, p, p, f64, i32, f64, i32, p, i32]
         L.orc_max_threads.argtypes = []
+        L.orc_visible_local.argtypes = [i64, f64, p]
+        L.orc_local_decode.argtypes = [i64, i64, i32, i32, p, p, p, p, p, p, p, f64, i32, f64, f64, p, i32]
         _lib = L
     return _lib
 
@@ -173,4 +175,33 @@ def masked_decode(kinds_list, pos_list, K_list, V_list, q, dtype: str, scale: fl
                                    kinds.ctypes.data, pos.ctypes.data, kv_off.ctypes.data, K.ctypes.data,
                                    V.ctypes.data, q.ctypes.data, scale, rot, base, policy, out.ctypes.data,
                                    n_threads), "masked_decode")
+    return out
+
+
+def visible_local(t_q: int, ratio: float) -> np.ndarray:
+    """Local Attention mask (Sec. 4.1): bool[t_q+1], the history indices the query at t_q sees."""
+    vis = np.empty(t_q + 1, dtype=np.uint8)
+    _check(lib().orc_visible_local(t_q, float(ratio), vis.ctypes.data), "visible_local")
+    return vis.astype(bool)
+
+
+def local_decode(pos_list, K_list, V_list, q, dtype: str, scale: float, ratio: float, rot: int = 0,
+                 base: float = 10000.0, n_threads: int = 0) -> np.ndarray:
+    """Decode under the Local Attention mask: the query of sequence s is its last history token."""
+    n_seq = len(pos_list)
+    H, d = q.shape[1], q.shape[2]
+    n_hist = _c([p.size for p in pos_list], np.int64)
+    hist_off = np.zeros(n_seq, dtype=np.int64)
+    hist_off[1:] = np.cumsum(n_hist)[:-1]
+    pos = _c(np.concatenate(pos_list), np.int32)
+    kv_sizes = np.array([k.size for k in K_list], dtype=np.int64)
+    kv_off = np.zeros(n_seq, dtype=np.int64)
+    kv_off[1:] = np.cumsum(kv_sizes)[:-1]
+    K = _c(np.concatenate([k.reshape(-1) for k in K_list]), np.uint16)
+    V = _c(np.concatenate([v.reshape(-1) for v in V_list]), np.uint16)
+    q = _c(q, np.uint16)
+    out = np.empty((n_seq, H, d), dtype=np.float64)
+    _check(lib().orc_local_decode(n_seq, H, d, _DT[dtype], n_hist.ctypes.data, hist_off.ctypes.data,
+                                  pos.ctypes.data, kv_off.ctypes.data, K.ctypes.data, V.ctypes.data, q.ctypes.data,
+                                  scale, rot, base, float(ratio), out.ctypes.data, n_threads), "local_decode")
     return out

@@ -394,3 +394,54 @@ int orc_max_threads(void) {
   return 1;
 #endif
 }
+
+/* ------------------------------------------------------------------------ */
+/* Local Attention baseline (Sec. 4.1 Baselines; Sec. 4.2: a FIFO queue of   */
+/* key-value memory at inference): token x_t (1-based t) attends within      */
+/* (floor(t*r), t].  With 0-based history indices, the query at index t_q     */
+/* sees j = floor((t_q + 1) * r) .. t_q (reading R14: the window closes on    */
+/* the query itself, as every causal mask does).                             */
+/* ------------------------------------------------------------------------ */
+
+int orc_visible_local(int64_t t_q, double ratio, uint8_t* vis) {
+  if (t_q < 0 || !(ratio >= 0.0) || !(ratio < 1.0)) return ORC_EINVAL;
+  const int64_t first = (int64_t)floor((double)(t_q + 1) * ratio); /* first visible index */
+  for (int64_t j = 0; j <= t_q; ++j) vis[j] = (uint8_t)(j >= first);
+  return ORC_OK;
+}
+
+/* Decode under the Local Attention mask over full histories (layout as orc_masked_decode). */
+int orc_local_decode(int64_t n_seq, int64_t H, int d, int dtype, const int64_t* n_hist, const int64_t* hist_off,
+                     const int32_t* pos, const int64_t* kv_off, const uint16_t* K, const uint16_t* V,
+                     const uint16_t* q, double scale, int rot, double base, double ratio, double* out,
+                     int n_threads) {
+  int rc_all = ORC_OK;
+#ifdef _OPENMP
+  if (n_threads > 0) omp_set_num_threads(n_threads);
+#else
+  (void)n_threads;
+#endif
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t sh = 0; sh < n_seq * H; ++sh) {
+    int64_t s = sh / H, h = sh % H;
+    int64_t T = n_hist[s];
+    uint8_t* vis = (uint8_t*)malloc((size_t)T);
+    int64_t* rows = (int64_t*)malloc(sizeof(int64_t) * (size_t)T);
+    int rc = (vis && rows) ? orc_visible_local(T - 1, ratio, vis) : ORC_ENOMEM;
+    if (rc == ORC_OK) {
+      int64_t n = 0;
+      for (int64_t j = 0; j < T; ++j)
+        if (vis[j]) rows[n++] = j;
+      const int32_t* ps = pos + hist_off[s];
+      rc = orc_attend(d, dtype, q + (s * H + h) * d, K + kv_off[s] + h * T * d, V + kv_off[s] + h * T * d, ps, rows,
+                      n, scale, rot, base, ps[T - 1], out + (s * H + h) * d);
+    }
+    if (rc != ORC_OK) {
+#pragma omp atomic write
+      rc_all = rc;
+    }
+    free(vis);
+    free(rows);
+  }
+  return rc_all;
+}

@@ -398,3 +398,40 @@ def test_rope_attention_depends_on_relative_positions_only():
     assert np.max(np.abs(a - b)) < 5e-3
     c = orc.masked_decode([kinds], [pos], [K], [V], q, "f16", 0.25, rot=0)[0, 0]
     assert np.max(np.abs(a - c)) > 1e-3  # the rotation is really applied
+
+
+# --------------------------------------------------------------------------
+# Local Attention baseline (Sec. 4.1)
+# --------------------------------------------------------------------------
+
+def test_local_window_closed_form_and_fifo_growth():
+    for r in (0.0, 0.3, 0.5, 0.75, 0.9):
+        prev_first = 0
+        for t in range(0, 400):
+            vis = orc.visible_local(t, r)
+            first = int(np.argmax(vis))
+            # 1-based x_{t+1} attends within (floor((t+1) r), t+1]: a contiguous window ending at the query
+            assert vis[t] and vis[first:].all() and not vis[:first].any()
+            assert first == math.floor((t + 1) * r)
+            # FIFO: the window's left end never moves back, and it admits exactly one new token per step
+            assert first >= prev_first
+            prev_first = first
+        # r = 0 is plain causal attention
+        assert orc.visible_local(57, 0.0).all()
+
+
+def test_local_decode_equals_sdpa_over_the_window():
+    rng = np.random.default_rng(13)
+    H, T, d = 2, 90, 16
+    K = _rand_bits(rng, (H, T, d))
+    V = _rand_bits(rng, (H, T, d))
+    q = _rand_bits(rng, (1, H, d))
+    pos = np.arange(T, dtype=np.int32)
+    for r in (0.0, 0.5, 0.8):
+        ours = orc.local_decode([pos], [K], [V], q, "f16", 0.4, r)[0]
+        first = math.floor(T * r)
+        Kt = torch.from_numpy(orc.decode16(K[:, first:], "f16"))
+        Vt = torch.from_numpy(orc.decode16(V[:, first:], "f16"))
+        qt = torch.from_numpy(orc.decode16(q[0], "f16")).unsqueeze(1)
+        ref = torch.nn.functional.scaled_dot_product_attention(qt, Kt, Vt, scale=0.4)[:, 0].numpy()
+        assert np.max(np.abs(ours - ref)) < 1e-12
