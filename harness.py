@@ -29,14 +29,21 @@ class StepInputs:
 
 class Runner:
     def __init__(self, w: wl.Workload, steps: int, policy: int = kvc.POLICY_PAPER, device=None,
-                 capacity_slack: int = 0, capacity=None):
+                 capacity_slack: int = 0, capacity=None, local_ratio: float = 0.0):
+        if w.extra.get("policy") == "local":  # the workload names its own cache policy
+            policy, local_ratio = kvc.POLICY_LOCAL, w.extra["local_ratio"]
         self.w = w
         self.steps = steps
         self.policy = policy
         self.device = torch.device("cuda", 0) if device is None else torch.device(device)
         self.tdt = torch.float16 if w.dtype == "f16" else torch.bfloat16
         cap = (w.capacity(steps) if capacity is None else np.asarray(capacity, np.int64)) + capacity_slack
-        self.cache = kvc.KVCache(w.M, w.H, w.d, cap, w.dtype, w.rotary_dim, w.rope_base, policy, device=self.device)
+        if policy == kvc.POLICY_LOCAL and capacity is None:
+            # a ring holding the largest window the run reaches: x_t sees (floor(t r), t]
+            T = w.prompt_len + steps
+            cap = T - np.floor(T * np.float64(np.float32(local_ratio))).astype(np.int64) + capacity_slack
+        self.cache = kvc.KVCache(w.M, w.H, w.d, cap, w.dtype, w.rotary_dim, w.rope_base, policy, device=self.device,
+                                 local_ratio=local_ratio)
         self.L = w.prompt_len.copy()
         self.open_cl = [-1] * w.b      # history index of an open <CL>
         self.g = 0                      # generated tokens so far

@@ -68,7 +68,11 @@ typedef enum {
    * enclosed rows and keeps <CR>.  Until then the open span's <CL> row is stored but skipped. */
   KVC_POLICY_PAPER = 0,
   /* Keeps <CL> (drops only the rows strictly between the sentinels) and shows it to later queries. */
-  KVC_POLICY_KEEP_CL = 1
+  KVC_POLICY_KEEP_CL = 1,
+  /* The paper's Local Attention baseline (Sec. 4.1; Sec. 4.2: a FIFO queue of key-value memory at
+   * inference): token x_t (1-based) attends within (floor(t * local_ratio), t].  The cache of a
+   * sequence is a ring of `capacity` rows that holds the window; no sentinel kinds are accepted. */
+  KVC_POLICY_LOCAL = 2
 } kvc_policy;
 
 const char* kvc_status_string(kvc_status s);
@@ -81,8 +85,11 @@ const char* kvc_last_error(void);
 
 typedef struct kvc_book kvc_book;
 
-/* b sequences; capacity[b] (host) bounds the rows each may store. */
+/* b sequences; capacity[b] (host) bounds the rows each may store.  For KVC_POLICY_LOCAL use
+ * kvc_book_create_local. */
 kvc_status kvc_book_create(int b, kvc_policy policy, const int64_t* capacity, kvc_book** out);
+/* A book of the Local Attention FIFO cache: each sequence's window must fit its capacity. */
+kvc_status kvc_book_create_local(int b, float local_ratio, const int64_t* capacity, kvc_book** out);
 void kvc_book_destroy(kvc_book* book);
 
 /* Tied positions (Sec. 3.1) of tokens about to be appended: n_new[b] tokens per sequence with
@@ -148,6 +155,7 @@ typedef struct {
   int32_t* orig_base;
   void* workspace;              /* device scratch owned by the cache while it lives */
   size_t workspace_bytes;
+  float local_ratio;            /* KVC_POLICY_LOCAL only: r in [0, 1); the window is ~(1 - r) of the history */
 } kvc_config;
 
 /* Byte sizes of the caller-owned buffers for `cfg` (k_base etc. may be NULL).  Any out pointer may

@@ -14,7 +14,7 @@ import numpy as np
 import synth
 from synth import workloads as wl
 
-from . import masked_decode, tied_positions, POLICY_PAPER
+from . import local_decode, masked_decode, tied_positions, POLICY_PAPER
 
 
 def history(w: wl.Workload, s: int, steps_done: int):
@@ -61,3 +61,20 @@ def expected_decode(w: wl.Workload, steps_done: int, layer: int, seqs, heads=Non
     q = np.stack(q_l)
     return masked_decode(kinds_l, pos_l, K_l, V_l, q, w.dtype, w.scale, rot=w.rotary_dim, base=w.rope_base,
                          policy=policy, n_threads=n_threads)
+
+
+def expected_local_decode(w: wl.Workload, steps_done: int, layer: int, seqs, ratio: float, heads=None,
+                          n_threads: int = 0) -> np.ndarray:
+    """fp64 decode under the Local Attention mask (the paper's Sec. 4.1 baseline) for the query at the
+    last token of each sequence's history; `ratio` as the cache holds it (a binary32 value)."""
+    pos_l, K_l, V_l, q_l = [], [], [], []
+    for s in seqs:
+        kinds, pos = history(w, s, steps_done)
+        T = kinds.size
+        K, V = kv_bits(w, layer, s, T, heads)
+        pos_l.append(pos)
+        K_l.append(K)
+        V_l.append(V)
+        q_l.append(q_bits(w, layer, s, T - 1, heads))
+    return local_decode(pos_l, K_l, V_l, np.stack(q_l), w.dtype, w.scale, ratio, rot=w.rotary_dim, base=w.rope_base,
+                        n_threads=n_threads)

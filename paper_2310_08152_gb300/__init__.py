@@ -18,7 +18,7 @@ import numpy as np
 from . import _lib
 
 NORMAL, CL, CR = 0, 1, 2
-POLICY_PAPER, POLICY_KEEP_CL = 0, 1
+POLICY_PAPER, POLICY_KEEP_CL, POLICY_LOCAL = 0, 1, 2
 F16, BF16 = 0, 1
 _DTYPES = {"f16": F16, "bf16": BF16}
 STATUS_NAMES = {0: "KVC_OK", 1: "KVC_ERR_INVALID_ARG", 2: "KVC_ERR_UNSUPPORTED", 3: "KVC_ERR_CAPACITY",
@@ -79,10 +79,13 @@ def _dev(t, name, dtype=None, numel=None):
 # span book (host only)
 # ------------------------------------------------------------------------------------------
 
-def kvc_book_create(b: int, capacity, policy: int = POLICY_PAPER) -> int:
+def kvc_book_create(b: int, capacity, policy: int = POLICY_PAPER, local_ratio: float = 0.0) -> int:
     cap = _np(capacity, np.int64)
     h = ctypes.c_void_p()
-    _check(lib().kvc_book_create(b, policy, cap.ctypes.data, ctypes.byref(h)))
+    if policy == POLICY_LOCAL:
+        _check(lib().kvc_book_create_local(b, float(local_ratio), cap.ctypes.data, ctypes.byref(h)))
+    else:
+        _check(lib().kvc_book_create(b, policy, cap.ctypes.data, ctypes.byref(h)))
     return h.value
 
 
@@ -159,11 +162,12 @@ class Book:
     A cache's own book (``KVCache.book``) is a read-only view: appends and compactions go through
     the cache so that its device state follows."""
 
-    def __init__(self, b: int, capacity, policy: int = POLICY_PAPER, _handle: Optional[int] = None):
+    def __init__(self, b: int, capacity, policy: int = POLICY_PAPER, _handle: Optional[int] = None,
+                 local_ratio: float = 0.0):
         self.b = b
         self._owned = _handle is None
         self.readonly = _handle is not None
-        self.handle = kvc_book_create(b, capacity, policy) if _handle is None else _handle
+        self.handle = kvc_book_create(b, capacity, policy, local_ratio) if _handle is None else _handle
 
     def next_positions(self, n_new, kinds):
         return kvc_book_next_positions(self.handle, n_new, kinds)
@@ -203,7 +207,8 @@ class Book:
 # cache
 # ------------------------------------------------------------------------------------------
 
-def make_config(M, H, d_head, capacity, dtype="f16", rotary_dim=0, rope_base=10000.0, policy=POLICY_PAPER):
+def make_config(M, H, d_head, capacity, dtype="f16", rotary_dim=0, rope_base=10000.0, policy=POLICY_PAPER,
+                local_ratio=0.0):
     cap = _np(capacity, np.int64)
     cfg = _lib.KvcConfig()
     cfg.M, cfg.H, cfg.d_head, cfg.b = M, H, d_head, cap.size
@@ -211,6 +216,7 @@ def make_config(M, H, d_head, capacity, dtype="f16", rotary_dim=0, rope_base=100
     cfg.rotary_dim = rotary_dim
     cfg.rope_base = rope_base
     cfg.policy = policy
+    cfg.local_ratio = local_ratio
     cfg.seq_capacity = cap.ctypes.data
     return cfg, cap
 
@@ -303,12 +309,13 @@ class KVCache:
     """A sentinel-compressed KV cache: owns its device buffers (torch) and the library handle."""
 
     def __init__(self, M: int, H: int, d_head: int, capacity, dtype: str = "f16", rotary_dim: int = 0,
-                 rope_base: float = 10000.0, policy: int = POLICY_PAPER, device=None):
+                 rope_base: float = 10000.0, policy: int = POLICY_PAPER, device=None, local_ratio: float = 0.0):
         import torch
 
         self.M, self.H, self.d, self.dtype = M, H, d_head, dtype
         self.rotary_dim, self.rope_base, self.policy = rotary_dim, rope_base, policy
-        cfg, cap = make_config(M, H, d_head, capacity, dtype, rotary_dim, rope_base, policy)
+        self.local_ratio = local_ratio
+        cfg, cap = make_config(M, H, d_head, capacity, dtype, rotary_dim, rope_base, policy, local_ratio)
         self.capacity = cap
         self.b = cap.size
         self.C = int(cap.sum())

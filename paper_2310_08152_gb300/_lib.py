@@ -29,6 +29,7 @@ class KvcConfig(ctypes.Structure):
         ("orig_base", P),
         ("workspace", P),
         ("workspace_bytes", c_size_t),
+        ("local_ratio", c_float),
     ]
 
 
@@ -37,6 +38,7 @@ SIGNATURES = [
     ("kvc_status_string", c_char_p, [c_int]),
     ("kvc_last_error", c_char_p, []),
     ("kvc_book_create", c_int, [c_int, c_int, P, P]),
+    ("kvc_book_create_local", c_int, [c_int, c_float, P, P]),
     ("kvc_book_destroy", None, [P]),
     ("kvc_book_next_positions", c_int, [P, P, P, P]),
     ("kvc_book_append", c_int, [P, P, P, P]),

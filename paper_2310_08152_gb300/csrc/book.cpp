@@ -2,11 +2,13 @@
 #include "book.hpp"
 
 #include <algorithm>
+#include <cmath>
 #include <cstdio>
 
 namespace kvc {
 
-Book::Book(int b, Policy policy, const int64_t* capacity) : b_(b), policy_(policy), seqs_(b) {
+Book::Book(int b, Policy policy, const int64_t* capacity, double local_ratio)
+    : b_(b), policy_(policy), local_ratio_(local_ratio), seqs_(b) {
   for (int s = 0; s < b; ++s) {
     seqs_[s].cap = capacity[s];
     seqs_[s].freed_before.push_back(0);
@@ -35,6 +37,13 @@ bool Book::check_append(const int32_t* n_new, const uint8_t* kinds, std::string&
         std::snprintf(buf, sizeof buf, "sequence %d token %d: kind %u is not NORMAL/CL/CR", s, t, k);
         err = buf;
         code = 1;
+        return false;
+      }
+      if (k != NORMAL && policy_ == POLICY_LOCAL) {
+        std::snprintf(buf, sizeof buf, "sequence %d token %d: sentinel kinds are not used by the local-attention "
+                      "cache", s, t);
+        err = buf;
+        code = 4;
         return false;
       }
       if (k == CL) {
@@ -69,7 +78,17 @@ bool Book::check_append(const int32_t* n_new, const uint8_t* kinds, std::string&
       stored_new = 0;
       for (int t = 0; t < n_new[s]; ++t) stored_new += kept[off + t];
     }
-    if (q.stored + stored_new > q.cap) {
+    if (policy_ == POLICY_LOCAL) {
+      const int64_t T = (int64_t)q.kind.size() + n_new[s];
+      const int64_t window = T > 0 ? T - local_first(T - 1) : 0;
+      if (window > q.cap) {
+        std::snprintf(buf, sizeof buf, "sequence %d: the local window of %lld rows exceeds capacity %lld", s,
+                      (long long)window, (long long)q.cap);
+        err = buf;
+        code = 3;
+        return false;
+      }
+    } else if (q.stored + stored_new > q.cap) {
       std::snprintf(buf, sizeof buf, "sequence %d: %lld stored + %lld new rows exceed capacity %lld", s,
                     (long long)q.stored, (long long)stored_new, (long long)q.cap);
       err = buf;
@@ -165,9 +184,19 @@ void Book::apply_append(const int32_t* n_new, const uint8_t* kinds, const int32_
       }
     }
     if (freed_any) rebuild_prefix(q);
-    q.stored += stored_new;
+    if (policy_ == POLICY_LOCAL) {
+      const int64_t T = (int64_t)q.kind.size();
+      q.stored = T > 0 ? T - local_first(T - 1) : 0;  // the window of the last token
+    } else {
+      q.stored += stored_new;
+    }
     off += n_new[s];
   }
+}
+
+int64_t Book::local_first(int64_t t) const {
+  // x_{t+1} (1-based) attends within (floor((t+1) r), t+1]: 0-based indices floor((t+1) r) .. t
+  return (int64_t)std::floor((double)(t + 1) * local_ratio_);
 }
 
 int Book::find_span(const Seq& q, int64_t cl) const {
@@ -278,6 +307,14 @@ bool Book::decode_view(int s, DecodeView& v, std::string& err) const {
   v.len = q.stored;
   v.qpos = q.pos.back();
   v.mask_lo = v.mask_hi = 0;
+  v.wrap = INT64_MAX;
+  if (policy_ == POLICY_LOCAL) {  // the window [first, tq] in ring slots
+    const int64_t first = local_first(tq);
+    v.begin = first % q.cap;
+    v.len = v.begin + (tq - first + 1);
+    v.wrap = q.cap - v.begin;
+    return true;
+  }
   if (q.kind[tq] == CL) {  // a <CL> attends only to itself (Sec. 3.1)
     v.begin = q.stored - 1;
     return true;
@@ -329,6 +366,11 @@ void Book::visible(int s, uint8_t* vis) const {
   const int64_t T = (int64_t)q.kind.size();
   if (T == 0) return;
   const int64_t tq = T - 1;
+  if (policy_ == POLICY_LOCAL) {
+    const int64_t first = local_first(tq);
+    for (int64_t j = 0; j < T; ++j) vis[j] = (uint8_t)(j >= first);
+    return;
+  }
   if (q.kind[tq] == CL) {
     for (int64_t j = 0; j < T; ++j) vis[j] = (uint8_t)(j == tq);
     return;
@@ -343,6 +385,14 @@ void Book::stored_rows(int s, std::vector<int32_t>& orig, std::vector<int32_t>& 
   const Seq& q = seqs_[s];
   orig.clear();
   pos.clear();
+  if (policy_ == POLICY_LOCAL) {  // the window of the last token, oldest first
+    const int64_t T = (int64_t)q.kind.size();
+    for (int64_t j = T > 0 ? local_first(T - 1) : 0; j < T; ++j) {
+      orig.push_back((int32_t)j);
+      pos.push_back(q.pos[j]);
+    }
+    return;
+  }
   for (int64_t j = 0; j < (int64_t)q.kind.size(); ++j) {
     if (stored_index(s, j) >= 0) {
       orig.push_back((int32_t)j);

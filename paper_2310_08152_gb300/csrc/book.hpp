@@ -15,7 +15,7 @@
 namespace kvc {
 
 enum Kind : uint8_t { NORMAL = 0, CL = 1, CR = 2 };
-enum Policy : int { POLICY_PAPER = 0, POLICY_KEEP_CL = 1 };
+enum Policy : int { POLICY_PAPER = 0, POLICY_KEEP_CL = 1, POLICY_LOCAL = 2 };
 
 struct Span {
   int64_t cl = -1;
@@ -24,11 +24,14 @@ struct Span {
 };
 
 // What a decode query of one sequence reads: stored rows [begin, len), except [mask_lo, mask_hi).
+// Under the local policy the rows live in a ring: row begin + r is slot begin + r for r < wrap and
+// slot r - wrap after it.
 struct DecodeView {
   int64_t len = 0;
   int64_t begin = 0;
   int64_t mask_lo = 0;
   int64_t mask_hi = 0;
+  int64_t wrap = INT64_MAX;
   int32_t qpos = 0;
   int64_t attended() const { return len - begin - (mask_hi - mask_lo); }
 };
@@ -44,13 +47,18 @@ struct CompactSeq {
 
 class Book {
  public:
-  Book(int b, Policy policy, const int64_t* capacity);
+  Book(int b, Policy policy, const int64_t* capacity, double local_ratio = 0.0);
 
   int b() const { return b_; }
   Policy policy() const { return policy_; }
   int64_t capacity(int s) const { return seqs_[s].cap; }
   int64_t stored(int s) const { return seqs_[s].stored; }
   int64_t history(int s) const { return (int64_t)seqs_[s].kind.size(); }
+  double local_ratio() const { return local_ratio_; }
+  // Local policy: first history index the query at t sees (the window is [local_first(t), t]).
+  int64_t local_first(int64_t t) const;
+  // Local policy: new token i of sequence s is written when it is among the last capacity tokens.
+  int64_t ring_slot(int s, int64_t j) const { return j % seqs_[s].cap; }
 
   // Validation only (no state change).  On error returns false and sets `err`.  With
   // free_in_block, the capacity check counts only the rows that will be stored.
@@ -97,6 +105,7 @@ class Book {
 
   int b_;
   Policy policy_;
+  double local_ratio_ = 0.0;
   std::vector<Seq> seqs_;
 };
 

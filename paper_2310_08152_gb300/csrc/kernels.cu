@@ -415,9 +415,11 @@ struct TileIter {
   int64_t x, hi, Lc, r;
   int s, h;
   __device__ __forceinline__ bool done() const { return x >= hi; }
-  __device__ __forceinline__ int n(int TR) const {
+  // rows of the next tile: at most TR, never past the segment, the range, or a ring's end (wrap)
+  __device__ __forceinline__ int n(int TR, int64_t wrap) const {
     int64_t k = Lc - r;
     if (hi - x < k) k = hi - x;
+    if (r < wrap && wrap - r < k) k = wrap - r;
     return (int)(k < TR ? k : TR);
   }
   __device__ __forceinline__ void advance(int n, const int64_t* P, int H) {
@@ -506,7 +508,8 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   // everything that depends only on the starting sequence, loaded together
   const int64_t P0 = p.P[ci.s], P1 = p.P[ci.s + 1];
   const DState ds0 = p.ds[ci.s];
-  int64_t seg_row0 = st.seq_row0[ci.s];  // issue side: row 0 of (s, h = 0) plus begin
+  int64_t seg_row0 = st.seq_row0[ci.s];  // issue side: row 0 of (s, h = 0)
+  int64_t seg_begin = ds0.begin, seg_wrap = ds0.wrap;
   int seg_cap = st.cap[ci.s];
   ci.Lc = P1 - P0;
   {
@@ -518,16 +521,19 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   ci.hi = hi;
   TileIter ii = ci;  // issued tiles (lane 0 uses it)
   int seg_s = ci.s;
-  seg_row0 += ds0.begin;
 
   auto issue = [&](int stage) {
-    const int n = ii.n(C::TR);
     if (ii.s != seg_s) {
       seg_s = ii.s;
-      seg_row0 = st.seq_row0[seg_s] + p.ds[seg_s].begin;
+      const DState d = p.ds[seg_s];
+      seg_row0 = st.seq_row0[seg_s];
+      seg_begin = d.begin;
+      seg_wrap = d.wrap;
       seg_cap = st.cap[seg_s];
     }
-    const int64_t row = seg_row0 + (int64_t)ii.h * seg_cap + ii.r;
+    const int n = ii.n(C::TR, seg_wrap);
+    const int64_t slot = ii.r < seg_wrap ? seg_begin + ii.r : ii.r - seg_wrap;
+    const int64_t row = seg_row0 + (int64_t)ii.h * seg_cap + slot;
     const uint32_t bytes = (uint32_t)n * L::RB;
     mbar_arrive_expect_tx(&full[stage], 2 * bytes);
     bulk_g2s(stg + stage * 2 * C::TILE, p.k + row * D, bytes, &full[stage]);
@@ -574,7 +580,7 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   const int rot = (L::A * grp + L::B * tl) % L::NV;
   float2 qv[L::EPL / 2], o[L::EPL / 2];
   float m = -INFINITY, l = 0.f;
-  int64_t mask_lo = ds0.mask_lo, mask_hi = ds0.mask_hi, begin = ds0.begin;
+  int64_t mask_lo = ds0.mask_lo, mask_hi = ds0.mask_hi, begin = ds0.begin, wrap = ds0.wrap;
   int32_t qpos = ds0.qpos;
   int cur_s = ci.s;
   bool dead = false;
@@ -584,16 +590,17 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   while (!ci.done()) {
     const int s = ci.s, h = ci.h;
     const int64_t r0 = ci.r;
-    const int n = ci.n(C::TR);
+    if (piece_start && s != cur_s) {  // the next sequence's state was prefetched with its q
+      cur_s = s;
+      mask_lo = dn.mask_lo;
+      mask_hi = dn.mask_hi;
+      begin = dn.begin;
+      wrap = dn.wrap;
+      qpos = dn.qpos;
+    }
+    const int n = ci.n(C::TR, wrap);
     const int stage = t % C::S;
     if (piece_start) {
-      if (s != cur_s) {  // the next sequence's state was prefetched with its q
-        cur_s = s;
-        mask_lo = dn.mask_lo;
-        mask_hi = dn.mask_hi;
-        begin = dn.begin;
-        qpos = dn.qpos;
-      }
       // stage q (rotated at the query position for RoPE, pre-scaled by scale*log2 e) in natural order
       const int half = g.rot / 2;
 #pragma unroll

@@ -8,9 +8,11 @@
 namespace kvc {
 
 // Per-sequence decode state, uploaded after every change of the span book.
-// The decode query of sequence s reads stored rows [begin, len) except [mask_lo, mask_hi).
+// The decode query of sequence s reads stored rows [begin, len) except [mask_lo, mask_hi).  Row
+// begin + r lives in slot begin + r while r < wrap and in slot r - wrap after it (a ring, for the
+// local-attention cache; wrap is INT32_MAX otherwise).
 struct DState {
-  int32_t len, begin, mask_lo, mask_hi, qpos, pad0, pad1, pad2;
+  int32_t len, begin, mask_lo, mask_hi, qpos, wrap, pad1, pad2;
 };
 
 // One stored token: its sequence, destination row, position, history index, and its index among

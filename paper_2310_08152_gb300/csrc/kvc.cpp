@@ -98,8 +98,10 @@ kvc_status check_config(const kvc_config* c, int64_t* C_out) {
     return fail(KVC_ERR_UNSUPPORTED, "rotary_dim=%d must be a multiple of 16 in [0, d_head]", c->rotary_dim);
   if (c->rotary_dim > 0 && !(c->rope_base > 1.0f))
     return fail(KVC_ERR_INVALID_ARG, "rope_base=%g must exceed 1", (double)c->rope_base);
-  if (c->policy != KVC_POLICY_PAPER && c->policy != KVC_POLICY_KEEP_CL)
+  if (c->policy != KVC_POLICY_PAPER && c->policy != KVC_POLICY_KEEP_CL && c->policy != KVC_POLICY_LOCAL)
     return fail(KVC_ERR_INVALID_ARG, "policy %d", (int)c->policy);
+  if (c->policy == KVC_POLICY_LOCAL && !(c->local_ratio >= 0.0f && c->local_ratio < 1.0f))
+    return fail(KVC_ERR_INVALID_ARG, "local_ratio=%g must be in [0, 1)", (double)c->local_ratio);
   if (!c->seq_capacity) return fail(KVC_ERR_INVALID_ARG, "seq_capacity is NULL");
   int64_t C = 0;
   for (int s = 0; s < c->b; ++s) {
@@ -185,7 +187,7 @@ class PinnedRing {
 
 struct kvc_book {
   kvc::Book book;
-  kvc_book(int b, kvc::Policy p, const int64_t* cap) : book(b, p, cap) {}
+  kvc_book(int b, kvc::Policy p, const int64_t* cap, double local_ratio = 0.0) : book(b, p, cap, local_ratio) {}
 };
 
 struct kvc_cache {
@@ -213,7 +215,8 @@ struct kvc_cache {
   bool last_was_decode = false;
   kvc::DecodePlan last_plan{-1, 0, 0, 0};
 
-  kvc_cache(const kvc_config& c, int64_t C_) : cfg(c), C(C_), bk(c.b, (kvc::Policy)c.policy, c.seq_capacity) {
+  kvc_cache(const kvc_config& c, int64_t C_)
+      : cfg(c), C(C_), bk(c.b, (kvc::Policy)c.policy, c.seq_capacity, (double)c.local_ratio) {
     cap.assign(c.seq_capacity, c.seq_capacity + c.b);
     off.resize(c.b);
     int64_t o = 0;
@@ -322,6 +325,7 @@ struct kvc_cache {
         ds[s].mask_lo = (int32_t)v.mask_lo;
         ds[s].mask_hi = (int32_t)v.mask_hi;
         ds[s].qpos = v.qpos;
+        ds[s].wrap = (int32_t)std::min<int64_t>(v.wrap, INT32_MAX);
         Lc = v.len - v.begin;
       } else {
         if (decode_ok) decode_err = err;
@@ -371,9 +375,21 @@ const char* kvc_last_error(void) { return g_last_error.c_str(); }
 // book
 // ------------------------------------------------------------------------------------------
 
+kvc_status kvc_book_create_local(int b, float local_ratio, const int64_t* capacity, kvc_book** out) {
+  if (!out || !capacity || b <= 0) return fail(KVC_ERR_INVALID_ARG, "b must be positive, pointers non-NULL");
+  if (!(local_ratio >= 0.0f && local_ratio < 1.0f)) return fail(KVC_ERR_INVALID_ARG, "local_ratio must be in [0, 1)");
+  for (int s = 0; s < b; ++s)
+    if (capacity[s] < 1) return fail(KVC_ERR_INVALID_ARG, "capacity[%d] < 1", s);
+  kvc_book* bk = new (std::nothrow) kvc_book(b, kvc::POLICY_LOCAL, capacity, (double)local_ratio);
+  if (!bk) return fail(KVC_ERR_NO_MEMORY, "book");
+  *out = bk;
+  return ok();
+}
+
 kvc_status kvc_book_create(int b, kvc_policy policy, const int64_t* capacity, kvc_book** out) {
   if (!out || !capacity || b <= 0) return fail(KVC_ERR_INVALID_ARG, "b must be positive, pointers non-NULL");
-  if (policy != KVC_POLICY_PAPER && policy != KVC_POLICY_KEEP_CL) return fail(KVC_ERR_INVALID_ARG, "policy");
+  if (policy != KVC_POLICY_PAPER && policy != KVC_POLICY_KEEP_CL)
+    return fail(KVC_ERR_INVALID_ARG, "policy %d (a local-attention book is made by kvc_book_create_local)", (int)policy);
   for (int s = 0; s < b; ++s)
     if (capacity[s] < 1) return fail(KVC_ERR_INVALID_ARG, "capacity[%d] < 1", s);
   kvc_book* bk = new (std::nothrow) kvc_book(b, (kvc::Policy)policy, capacity);
@@ -562,10 +578,21 @@ static kvc_status append_impl(kvc_cache* c, int layer, const void* k, const void
   if (starts) {
     int64_t N = 0;
     for (int s = 0; s < c->cfg.b; ++s) N += n_new[s];
+    const bool local = c->cfg.policy == KVC_POLICY_LOCAL;
     std::vector<uint8_t> kept;
-    if (free_in_block) c->bk.book.kept_in_block(n_new, kinds, kept);
+    if (free_in_block && !local) {
+      c->bk.book.kept_in_block(n_new, kinds, kept);
+    } else if (local) {  // a ring: only the last `capacity` new tokens of a sequence survive the call
+      kept.assign((size_t)N, 1);
+      int64_t o = 0;
+      for (int s = 0; s < c->cfg.b; ++s) {
+        for (int i = 0; i < n_new[s] - c->cap[s]; ++i) kept[o + i] = 0;
+        o += n_new[s];
+      }
+    }
+    const bool filtered = !kept.empty();
     int64_t n_plan = 0;
-    for (int64_t t = 0; t < N; ++t) n_plan += free_in_block ? kept[t] : 1;
+    for (int64_t t = 0; t < N; ++t) n_plan += filtered ? kept[t] : 1;
     // destination rows before the book moves on
     std::vector<int64_t> row0(c->cfg.b), orig0(c->cfg.b);
     for (int s = 0; s < c->cfg.b; ++s) {
@@ -576,16 +603,16 @@ static kvc_status append_impl(kvc_cache* c, int layer, const void* k, const void
     cudaError_t e;
     unsigned char* img = c->ring.reserve(bytes, &e);
     if (!img) return cuda_fail(e, "staging");
-    c->bk.book.apply_append(n_new, kinds, pos, free_in_block ? kept.data() : nullptr);
+    c->bk.book.apply_append(n_new, kinds, pos, (free_in_block && !local) ? kept.data() : nullptr);
     c->fill_state(img);
     kvc::TokPlan* tp = reinterpret_cast<kvc::TokPlan*>(img + c->ws.dyn_payload);
     int64_t t = 0, w = 0;
     for (int s = 0; s < c->cfg.b; ++s) {
       int64_t row = row0[s];
       for (int i = 0; i < n_new[s]; ++i, ++t) {
-        if (free_in_block && !kept[t]) continue;  // freed as it is written: never stored
+        if (filtered && !kept[t]) continue;  // freed as it is written (or overtaken in the ring): never stored
         tp[w].s = s;
-        tp[w].row = (int32_t)row++;
+        tp[w].row = local ? (int32_t)((orig0[s] + i) % c->cap[s]) : (int32_t)row++;
         tp[w].pos = pos[t];
         tp[w].orig = (int32_t)(orig0[s] + i);
         tp[w].in_tok = (int32_t)t;
@@ -781,6 +808,23 @@ kvc_status kvc_masked_reference_layout(kvc_cache* c, int seq, int64_t cap, uint8
   st = c->ensure_cuda(stream);
   if (st != KVC_OK) return st;
   cudaError_t e = cudaSuccess;
+  if (c->cfg.policy == KVC_POLICY_LOCAL) {  // the window, oldest first, out of the ring
+    const int64_t cap = c->cap[seq];
+    std::vector<int32_t> o((size_t)cap), p((size_t)cap);
+    e = cudaMemcpyAsync(o.data(), c->cfg.orig_base + c->off[seq], 4 * (size_t)cap, cudaMemcpyDeviceToHost, stream);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(p.data(), c->cfg.pos_base + c->off[seq], 4 * (size_t)cap, cudaMemcpyDeviceToHost, stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return cuda_fail(e, "read back stored rows");
+    const int64_t T = c->bk.book.history(seq);
+    const int64_t first = c->bk.book.local_first(T - 1);
+    for (int64_t k = 0; k < ns; ++k) {
+      const int64_t slot = (first + k) % cap;
+      if (stored_orig_idx) stored_orig_idx[k] = o[(size_t)slot];
+      if (stored_pos) stored_pos[k] = p[(size_t)slot];
+    }
+    return ok();
+  }
   if (stored_orig_idx)
     e = cudaMemcpyAsync(stored_orig_idx, c->cfg.orig_base + c->off[seq], 4 * (size_t)ns, cudaMemcpyDeviceToHost,
                         stream);

@@ -167,6 +167,20 @@ def opt13b_uncompressed(b: int = 16, L: int = 2048, M: int = 24) -> Workload:
                     note=f"OPT-1.3B-shaped, no spans (r=0): M={M}, H=32, d=64, fp16, b={b}, L={L}")
 
 
+def opt13b_local(ratio: float = 0.5, b: int = 16, L: int = 2048, M: int = 24) -> Workload:
+    """The paper's Local Attention baseline (Sec. 4.1; FIFO queue at inference, Sec. 4.2) on the
+    OPT-1.3B-shaped cache: no sentinels, each token attends within a window of ~(1 - r) of its
+    history.  At r = 0.5 it keeps as many rows as the compressed cache with 32 of 64 tokens enclosed."""
+    kinds = np.zeros(L, dtype=np.uint8)
+    w = Workload(f"opt1.3b_local{ratio:g}", 1, M=M, H=32, d=64, dtype="f16", b=b,
+                 prompt_kinds=[kinds.copy() for _ in range(b)], prompt_spans=[[] for _ in range(b)], n_steps=128,
+                 gen_kind=_normal_gen, scale=1.0 / math.sqrt(64), seed=SEED_BASE + 1,
+                 note=f"OPT-1.3B-shaped Local Attention FIFO cache (r={ratio:g}): M={M}, H=32, d=64, fp16, b={b}, "
+                      f"L={L}")
+    w.extra = {"policy": "local", "local_ratio": ratio}
+    return w
+
+
 def opt27b(b: int = 32, L: int = 4096, M: int = 32) -> Workload:
     kinds, spans = block_kinds(L, 44)
     return Workload("opt2.7b", 2, M=M, H=32, d=80, dtype="bf16", b=b, prompt_kinds=[kinds.copy() for _ in range(b)],
@@ -233,7 +247,7 @@ def throughput_3b(ratio: float, b: int, prefix: int = 800, M: int = 32, steps: i
 
 def by_name(name: str, **kw) -> Workload:
     table = {"tiny": tiny, "opt1.3b": opt13b, "opt1.3b_r0": opt13b_uncompressed, "opt2.7b": opt27b,
-             "ragged": ragged}
+             "ragged": ragged, "opt1.3b_local0.5": opt13b_local}
     if name.startswith("rope3b"):
         interior = int(name.split("_I")[1]) if "_I" in name else 32
         return rope3b(interior=interior, **kw)

@@ -295,3 +295,35 @@ def test_write_time_freeing_capacity_counts_stored_rows():
     book.append([9], [NORMAL, CL, NORMAL, NORMAL, NORMAL, NORMAL, CR, NORMAL, NORMAL], free_closed=True)
     assert book.lengths()[0][0] == 4
     assert _err(book.append, [2], [NORMAL, NORMAL]) == 3
+
+
+@pytest.mark.parametrize("ratio", [0.0, 0.3, 0.5, 0.8])
+def test_local_book_window_matches_oracle(ratio):
+    """The Local Attention FIFO cache (Sec. 4.1/4.2) keeps exactly the window the mask shows."""
+    rng = np.random.default_rng(22)
+    r32 = float(np.float32(ratio))
+    cap = np.array([700, 700], np.int64)
+    book = kvc.Book(2, cap, kvc.POLICY_LOCAL, local_ratio=ratio)
+    T = [0, 0]
+    for _ in range(25):
+        n_new = rng.integers(0, 30, size=2).astype(np.int32)
+        book.append(n_new, np.zeros(int(n_new.sum()), np.uint8))
+        ln, at = book.lengths()
+        for s in range(2):
+            T[s] += int(n_new[s])
+            if not T[s]:
+                continue
+            vis = orc.visible_local(T[s] - 1, r32)
+            lay = book.layout(s)
+            assert np.array_equal(lay["visible"], vis)
+            assert np.array_equal(lay["stored_orig"], np.nonzero(vis)[0])
+            assert ln[s] == at[s] == vis.sum()
+    assert _err(book.append, [1, 0], [CL]) == 4  # no sentinels in a local-attention cache
+
+
+def test_local_book_capacity_is_the_window():
+    book = kvc.Book(1, [10], kvc.POLICY_LOCAL, local_ratio=0.5)
+    book.append([19], np.zeros(19, np.uint8))  # x_19 sees (9, 19]: 10 rows
+    assert book.lengths()[0][0] == 10
+    book.append([1], [NORMAL])  # x_20 sees (10, 20]: still 10
+    assert _err(book.append, [2], [NORMAL, NORMAL]) == 3  # x_22 would see (11, 22]: 11 rows

@@ -261,3 +261,28 @@ def test_write_time_freeing_prompt_modes(mode, block):
             for m in range(w.M):
                 compare(out[m].cpu().numpy(), ow.expected_decode(w, g + 1, m, list(range(w.b))), f"{mode} {g} {m}")
         assert run.cache.device_status() == 0
+
+
+@pytest.mark.parametrize("ratio", [0.5, 0.8, 0.0])
+def test_local_attention_fifo_cache(ratio):
+    # the paper's Local Attention baseline (Sec. 4.1; FIFO queue at inference, Sec. 4.2): a ring per
+    # (layer, K/V, head), decode over the window, compared with the oracle's local mask
+    for w in (wl.opt13b_uncompressed(b=3, L=700, M=2), dataclasses.replace(wl.rope3b(32, b=2, L=300, M=1),
+                                                                           prompt_kinds=[np.zeros(300, np.uint8)] * 2,
+                                                                           prompt_spans=[[], []], name="rope-local")):
+        run = harness.Runner(w, steps=6, policy=kvc.POLICY_LOCAL, local_ratio=ratio)
+        run.load_prompt()
+        out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device="cuda")
+        r32 = float(np.float32(ratio))
+        for g in range(6):
+            run.step(run.make_step_inputs(g), out)
+            torch.cuda.synchronize()
+            for m in range(w.M):
+                ref = ow.expected_local_decode(w, g + 1, m, list(range(w.b)), r32)
+                compare(out[m].cpu().numpy(), ref, f"local r={ratio} step {g} layer {m}")
+            for s in range(w.b):
+                lay = run.cache.masked_reference_layout(s)
+                T = lay["kinds"].size
+                first = int(np.floor(T * np.float64(r32)))
+                assert np.array_equal(lay["stored_orig"], np.arange(first, T))
+        assert run.cache.device_status() == 0
