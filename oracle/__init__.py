@@ -55,6 +55,8 @@ def lib():
         L.orc_max_threads.argtypes = []
         L.orc_visible_local.argtypes = [i64, f64, p]
         L.orc_local_decode.argtypes = [i64, i64, i32, i32, p, p, p, p, p, p, p, f64, i32, f64, f64, p, i32]
+        L.orc_masked_prefill.argtypes = [i64, i64, i32, i32, p, p, p, p, p, p, p, p, p, p, f64, i32, f64, i32, p,
+                                         i32]
         _lib = L
     return _lib
 
@@ -204,4 +206,38 @@ def local_decode(pos_list, K_list, V_list, q, dtype: str, scale: float, ratio: f
     _check(lib().orc_local_decode(n_seq, H, d, _DT[dtype], n_hist.ctypes.data, hist_off.ctypes.data,
                                   pos.ctypes.data, kv_off.ctypes.data, K.ctypes.data, V.ctypes.data, q.ctypes.data,
                                   scale, rot, base, float(ratio), out.ctypes.data, n_threads), "local_decode")
+    return out
+
+
+def masked_prefill(kinds_list, pos_list, K_list, V_list, n_q, Q, dtype: str, scale: float, rot: int = 0,
+                   base: float = 10000.0, policy: int = POLICY_PAPER, n_threads: int = 0) -> np.ndarray:
+    """Prefill under the sentinel mask: sequence s's queries are its last n_q[s] history tokens.
+
+    kinds_list/pos_list/K_list/V_list as ``masked_decode``; Q: uint16 [sum n_q, H, d] (sequence s's
+    queries consecutive, oldest first).  Returns fp64 [sum n_q, H, d].
+    """
+    n_seq = len(kinds_list)
+    H, d = Q.shape[1], Q.shape[2]
+    n_hist = _c([k.size for k in kinds_list], np.int64)
+    hist_off = np.zeros(n_seq, dtype=np.int64)
+    hist_off[1:] = np.cumsum(n_hist)[:-1]
+    n_q = _c(n_q, np.int64)
+    assert n_q.size == n_seq and Q.shape[0] == int(n_q.sum())
+    q_off = np.zeros(n_seq, dtype=np.int64)
+    q_off[1:] = np.cumsum(n_q)[:-1]
+    kinds = _c(np.concatenate(kinds_list), np.uint8)
+    pos = _c(np.concatenate(pos_list), np.int32)
+    for s in range(n_seq):
+        assert K_list[s].shape == (H, n_hist[s], d) and V_list[s].shape == (H, n_hist[s], d)
+    kv_sizes = np.array([k.size for k in K_list], dtype=np.int64)
+    kv_off = np.zeros(n_seq, dtype=np.int64)
+    kv_off[1:] = np.cumsum(kv_sizes)[:-1]
+    K = _c(np.concatenate([k.reshape(-1) for k in K_list]), np.uint16)
+    V = _c(np.concatenate([v.reshape(-1) for v in V_list]), np.uint16)
+    Q = _c(Q, np.uint16)
+    out = np.empty(Q.shape, dtype=np.float64)
+    _check(lib().orc_masked_prefill(n_seq, H, d, _DT[dtype], n_hist.ctypes.data, hist_off.ctypes.data,
+                                    kinds.ctypes.data, pos.ctypes.data, kv_off.ctypes.data, K.ctypes.data,
+                                    V.ctypes.data, n_q.ctypes.data, q_off.ctypes.data, Q.ctypes.data, scale, rot,
+                                    base, policy, out.ctypes.data, n_threads), "masked_prefill")
     return out

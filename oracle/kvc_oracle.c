@@ -17,6 +17,8 @@
  *   - single-query softmax attention over a set of rows, in fp64  (Sec. 2, Complexity of Attention)
  *   - RoPE (rotate-half convention) for the rotary configuration  (Sec. 1 cites rotary encoding; the
  *                                                                  convention is a reading, see below)
+ *   - masked prefill: every query of a prompt block under the mask (Sec. 3.1)
+ *   - the Local Attention baseline's window                       (Sec. 4.1 Baselines, Sec. 4.2)
  *
  * Readings of points the paper leaves open (each is also listed in the design notes):
  *   R1 <CL> is never visible to later queries under POLICY_PAPER (normal tokens see only "previous
@@ -435,6 +437,63 @@ int orc_local_decode(int64_t n_seq, int64_t H, int d, int dtype, const int64_t* 
       const int32_t* ps = pos + hist_off[s];
       rc = orc_attend(d, dtype, q + (s * H + h) * d, K + kv_off[s] + h * T * d, V + kv_off[s] + h * T * d, ps, rows,
                       n, scale, rot, base, ps[T - 1], out + (s * H + h) * d);
+    }
+    if (rc != ORC_OK) {
+#pragma omp atomic write
+      rc_all = rc;
+    }
+    free(vis);
+    free(rows);
+  }
+  return rc_all;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Masked prefill (Sec. 3.1: the modified mask holds for every token of a    */
+/* prompt in the forward pass; Manipulating Key-Value Memory: a long prefix  */
+/* may be run block by block).  For sequence s the queries are its last      */
+/* n_q[s] history tokens; the query at history index t attends to [0, t]     */
+/* under orc_visible(t) -- the same rows a decode step at t would see.       */
+/*   kinds/pos/K/V: as orc_masked_decode                                     */
+/*   Q:   [sum n_q][H][d], sequence s's queries from row q_off[s], oldest    */
+/*        first; out: same layout, fp64.                                     */
+/* ------------------------------------------------------------------------ */
+
+int orc_masked_prefill(int64_t n_seq, int64_t H, int d, int dtype, const int64_t* n_hist, const int64_t* hist_off,
+                       const uint8_t* kinds, const int32_t* pos, const int64_t* kv_off, const uint16_t* K,
+                       const uint16_t* V, const int64_t* n_q, const int64_t* q_off, const uint16_t* Q,
+                       double scale, int rot, double base, int policy, double* out, int n_threads) {
+  int64_t n_items = 0;
+  for (int64_t s = 0; s < n_seq; ++s) {
+    if (n_q[s] < 0 || n_q[s] > n_hist[s]) return ORC_EINVAL;
+    n_items += n_q[s];
+  }
+  int rc_all = ORC_OK;
+#ifdef _OPENMP
+  if (n_threads > 0) omp_set_num_threads(n_threads);
+#else
+  (void)n_threads;
+#endif
+#pragma omp parallel for schedule(dynamic, 4)
+  for (int64_t it = 0; it < n_items; ++it) {
+    /* item -> (sequence, query) by a linear walk: plain, and cheap beside the attention */
+    int64_t s = 0, i = it;
+    while (i >= n_q[s]) i -= n_q[s++];
+    const int64_t T = n_hist[s];
+    const int64_t t = T - n_q[s] + i; /* the query's history index */
+    uint8_t* vis = (uint8_t*)malloc((size_t)(t + 1));
+    int64_t* rows = (int64_t*)malloc(sizeof(int64_t) * (size_t)(t + 1));
+    int rc = (vis && rows) ? orc_visible(kinds + hist_off[s], t, policy, vis) : ORC_ENOMEM;
+    if (rc == ORC_OK) {
+      int64_t n = 0;
+      for (int64_t j = 0; j <= t; ++j)
+        if (vis[j]) rows[n++] = j;
+      const int32_t* ps = pos + hist_off[s];
+      for (int64_t h = 0; h < H && rc == ORC_OK; ++h) {
+        const int64_t qrow = (q_off[s] + i) * H + h;
+        rc = orc_attend(d, dtype, Q + qrow * d, K + kv_off[s] + h * T * d, V + kv_off[s] + h * T * d, ps, rows, n,
+                        scale, rot, base, ps[t], out + qrow * d);
+      }
     }
     if (rc != ORC_OK) {
 #pragma omp atomic write

@@ -435,3 +435,95 @@ def test_local_decode_equals_sdpa_over_the_window():
         qt = torch.from_numpy(orc.decode16(q[0], "f16")).unsqueeze(1)
         ref = torch.nn.functional.scaled_dot_product_attention(qt, Kt, Vt, scale=0.4)[:, 0].numpy()
         assert np.max(np.abs(ours - ref)) < 1e-12
+
+
+# --------------------------------------------------------------------------
+# Masked prefill (Sec. 3.1: the mask over every token of a prompt block)
+# --------------------------------------------------------------------------
+
+def _sdpa(q, k, v, scale, mask=None, causal=False):
+    """fp64 library attention: q [H, Tq, d], k/v [H, Tk, d]."""
+    return torch.nn.functional.scaled_dot_product_attention(
+        torch.from_numpy(q), torch.from_numpy(k), torch.from_numpy(v), scale=scale,
+        attn_mask=None if mask is None else torch.from_numpy(mask), is_causal=causal).numpy()
+
+
+@pytest.mark.parametrize("dtype", ["f16", "bf16"])
+def test_prefill_spanfree_equals_causal_sdpa(dtype):
+    """No spans: every query of the block is plain causal attention (library routine)."""
+    rng = np.random.default_rng(21)
+    H, d, scale = 3, 16, 0.35
+    Ts, nqs = [70, 41], [70, 13]
+    kinds_l = [np.zeros(T, np.uint8) for T in Ts]
+    pos_l = [orc.tied_positions(k) for k in kinds_l]
+    K_l = [_rand_bits(rng, (H, T, d), dtype) for T in Ts]
+    V_l = [_rand_bits(rng, (H, T, d), dtype) for T in Ts]
+    Q_full = [_rand_bits(rng, (T, H, d), dtype) for T in Ts]
+    Q = np.concatenate([q[T - n:] for q, T, n in zip(Q_full, Ts, nqs)])
+    ours = orc.masked_prefill(kinds_l, pos_l, K_l, V_l, nqs, Q, dtype, scale)
+    row = 0
+    for s, (T, n) in enumerate(zip(Ts, nqs)):
+        qf = orc.decode16(Q_full[s], dtype).transpose(1, 0, 2)  # [H, T, d]
+        ref = _sdpa(qf, orc.decode16(K_l[s], dtype), orc.decode16(V_l[s], dtype), scale, causal=True)
+        got = ours[row:row + n].transpose(1, 0, 2)
+        assert np.max(np.abs(got - ref[:, T - n:])) < 1e-12
+        row += n
+
+
+@pytest.mark.parametrize("policy", [orc.POLICY_PAPER, orc.POLICY_KEEP_CL])
+@pytest.mark.parametrize("rot", [0, 16])
+def test_prefill_equals_sdpa_with_the_mask_matrix(policy, rot):
+    """With spans (closed, open, at the block's edges) and RoPE: the block's outputs equal library
+    attention with a boolean mask whose row t is the query-t mask, on keys rotated at their tied
+    positions and rounded to the cache type, and queries rotated at theirs."""
+    rng = np.random.default_rng(22 + rot + policy)
+    H, d, scale, base = 2, 16, 0.3, 10000.0
+    kinds_l = [np.concatenate([wl.block_kinds(128, 20)[0], _random_wellformed(rng, 61)]),
+               _random_wellformed(rng, 97, p_open=0.3, p_close=0.3)]
+    nqs = [100, 97]
+    pos_l = [orc.tied_positions(k) for k in kinds_l]
+    K_l = [_rand_bits(rng, (H, k.size, d)) for k in kinds_l]
+    V_l = [_rand_bits(rng, (H, k.size, d)) for k in kinds_l]
+    Q_full = [_rand_bits(rng, (k.size, H, d)) for k in kinds_l]
+    Q = np.concatenate([q[q.shape[0] - n:] for q, n in zip(Q_full, nqs)])
+    ours = orc.masked_prefill(kinds_l, pos_l, K_l, V_l, nqs, Q, "f16", scale, rot=rot, base=base, policy=policy)
+    row = 0
+    for s, kinds in enumerate(kinds_l):
+        T, n = kinds.size, nqs[s]
+        mask = np.zeros((n, T), dtype=bool)
+        for i in range(n):
+            t = T - n + i
+            mask[i, :t + 1] = orc.visible(kinds[:t + 1], t, policy)
+        pos = pos_l[s]
+        kf = orc.decode16(K_l[s], "f16")
+        qf = orc.decode16(Q_full[s][T - n:], "f16").transpose(1, 0, 2)
+        if rot:
+            kf = np.stack([[orc.decode16(orc.encode16(orc.rope(kf[h, j], rot, base, pos[j]), "f16"), "f16")
+                            for j in range(T)] for h in range(H)])
+            qf = np.stack([[orc.rope(qf[h, i], rot, base, pos[T - n + i]) for i in range(n)] for h in range(H)])
+        ref = _sdpa(qf, kf, orc.decode16(V_l[s], "f16"), scale, mask=mask)
+        got = ours[row:row + n].transpose(1, 0, 2)
+        assert np.max(np.abs(got - ref)) < 1e-12
+        # Sec. 3.1: a <CL> query attends only to itself -> exactly its value row
+        for i in range(n):
+            if kinds[T - n + i] == CL:
+                assert np.array_equal(got[:, i], orc.decode16(V_l[s][:, T - n + i], "f16"))
+        row += n
+    assert any((k == CL).any() for k in kinds_l)
+
+
+def test_prefill_row_equals_decode_at_its_prefix():
+    """Query t of a prefill block is the decode step whose history ends at t."""
+    rng = np.random.default_rng(23)
+    H, d = 2, 8
+    kinds = np.concatenate([wl.block_kinds(64, 30)[0], np.uint8([NORMAL, CL, NORMAL, NORMAL, CR, NORMAL])])
+    T = kinds.size
+    pos = orc.tied_positions(kinds)
+    K = _rand_bits(rng, (H, T, d))
+    V = _rand_bits(rng, (H, T, d))
+    Q = _rand_bits(rng, (T, H, d))
+    pre = orc.masked_prefill([kinds], [pos], [K], [V], [T], Q, "f16", 0.6, rot=8)
+    for t in (0, 6, 7, 8, 38, 39, 40, 63, 64, 65, 66, 68, 69):
+        dec = orc.masked_decode([kinds[:t + 1]], [pos[:t + 1]], [K[:, :t + 1]], [V[:, :t + 1]], Q[t:t + 1], "f16",
+                                0.6, rot=8)[0]
+        assert np.array_equal(pre[t], dec)
