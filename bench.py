@@ -63,9 +63,11 @@ def measured_hbm_peak():
 
 def kernel_source_hash() -> str:
     """Hash of the decode kernel's source: its device helpers, the kernel and its launcher."""
-    text = open(os.path.join(ROOT, "paper_2310_08152_gb300/csrc/kernels.cu")).read()
-    marks = [("// RoPE angle.", "// a1: append"), ("// a5 + a6: decode", "cudaError_t launch_append_t")]
+    csrc = os.path.join(ROOT, "paper_2310_08152_gb300/csrc")
+    text = open(os.path.join(csrc, "kernels.cu")).read()
+    marks = [("// a5 + a6: decode", "cudaError_t launch_append_t")]
     h = hashlib.sha256()
+    h.update(open(os.path.join(csrc, "device_common.cuh")).read().encode())
     for a, b in marks:
         i = text.index(a)
         h.update(text[i:text.index(b, i)].encode())

@@ -120,6 +120,63 @@ class Runner:
                 timer.append(ev)
         del kbuf, vbuf
 
+    def prefill_prompt(self, block: int = 0, stream=None, out_cb=None, layers=None, events=None):
+        """Prompt ingestion with masked prefill attention (Sec. 3.1): per block of `block` tokens of
+        every sequence (0: the whole prompt in one go), append the block's K/V layer by layer, run the
+        prefill of that layer's queries (the block's tokens) over the stored rows, and once every layer
+        is written free the spans closed so far -- the paper's for-loop over blocks.
+
+        out_cb(start, n, layer, out): receives each prefilled layer's output, fp32 [sum n, H, d]
+        (sequence-major).  events: a list that receives a (start, end) CUDA event pair around each
+        prefill call."""
+        w = self.w
+        start = np.zeros(w.b, np.int64)
+        while (start < self.L).any():
+            n = self.L - start if block <= 0 else np.minimum(self.L - start, block)
+            self._prefill_block(start, n, stream, out_cb, layers, events)
+            start = start + n
+            seq, cl, cr = [], [], []
+            for s in range(w.b):
+                for a, c in self.cache.pending_spans(s):
+                    seq.append(s)
+                    cl.append(a)
+                    cr.append(c)
+            if seq:
+                self.cache.compress_spans(seq, cl, cr, stream)
+
+    def _prefill_block(self, start, n, stream, out_cb, layers, events):
+        w = self.w
+        n_new = n.astype(np.int32)
+        kinds = np.concatenate([w.prompt_kinds[s][start[s]:start[s] + n[s]] for s in range(w.b)]).astype(np.uint8)
+        N = int(n_new.sum())
+        tok_t = torch.from_numpy(np.concatenate([np.arange(start[s], start[s] + n[s], dtype=np.int32)
+                                                 for s in range(w.b)])).to(self.device)
+        tok_s = torch.from_numpy(np.repeat(np.arange(w.b, dtype=np.int32), n)).to(self.device)
+        kbuf = torch.empty(N * w.H * w.d, dtype=self.tdt, device=self.device)
+        vbuf = torch.empty_like(kbuf)
+        qbuf = torch.empty_like(kbuf)
+        out = torch.empty(N, w.H, w.d, dtype=torch.float32, device=self.device)
+        for m in range(w.M):
+            self._fill(synth.K_TENSOR, m, tok_t, tok_s, kbuf, self.kv_scale)
+            self._fill(synth.V_TENSOR, m, tok_t, tok_s, vbuf, self.kv_scale)
+            if m == 0:
+                pos = self.cache.book.next_positions(n_new, kinds)
+                kvc.kvc_append(self.cache.handle, 0, kbuf, vbuf, n_new, pos, kinds, stream)
+            else:
+                kvc.kvc_append(self.cache.handle, m, kbuf, vbuf, None, None, None, stream)
+            if layers is not None and m not in layers:
+                continue
+            self._fill(synth.Q_TENSOR, m, tok_t, tok_s, qbuf, self.q_scale)
+            if events is not None:
+                ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                ev[0].record(stream)
+            kvc.kvc_prefill_attention(self.cache.handle, m, qbuf, n_new, w.scale, out, stream)
+            if events is not None:
+                ev[1].record(stream)
+                events.append(ev)
+            if out_cb is not None:
+                out_cb(start, n, m, out)
+
     def compress_prompt(self, stream=None):
         seq, cl, cr = [], [], []
         for s in range(self.w.b):

@@ -16,6 +16,7 @@
  *   kvc_append            write new tokens' K/V rows and their positions      (Sec. 2; Sec. 3.1 positions)
  *   kvc_compress_spans    free the rows of closed spans by in-place compaction (Sec. 3.1, freeing the KV)
  *   kvc_decode_attention  one query per (sequence, head) over the kept rows    (Sec. 1 / 3.1 mask; Sec. 4.3)
+ *   kvc_prefill_attention every query of a prompt block under the mask, on tensor cores (Sec. 3.1)
  *   kvc_masked_reference_layout   the full history, the mask and the stored rows, for verification
  * plus a host-only span book (kvc_book_*) holding the span bookkeeping that
  * decides what each call does.
@@ -116,6 +117,16 @@ kvc_status kvc_book_compress(kvc_book* book, const int32_t* seq, const int64_t* 
 /* Closed spans of `seq` that are not yet freed: up to `max` (cl, cr) pairs; *n gets the count. */
 kvc_status kvc_book_pending_spans(const kvc_book* book, int seq, int64_t* cl, int64_t* cr, int64_t max,
                                   int64_t* n);
+
+/* Mask bounds of the masked prefill (kvc_prefill_attention) of the last n_q tokens of `seq`: for
+ * each stored row i (up to `max`; *n gets the stored-row count) meta[i] = (hid << 1) | is_cl, where
+ * row i is visible to the query at stored row iq exactly when i <= iq <= hid, except that a query
+ * whose own row has is_cl set (a <CL>, Sec. 3.1) sees only itself.  hid is the stored row of the
+ * <CR> that closes a span enclosing row i, i itself for a <CL> row under KVC_POLICY_PAPER, and
+ * 0x3FFFFFFF otherwise.  KVC_ERR_STATE if the last n_q tokens are not all stored rows;
+ * KVC_ERR_UNSUPPORTED under KVC_POLICY_LOCAL. */
+kvc_status kvc_book_prefill_keys(const kvc_book* book, int seq, int64_t n_q, int32_t* meta, int64_t max,
+                                 int64_t* n);
 
 /* Stored rows per sequence (len_out[b]) and rows the next decode attends to (attend_out[b]);
  * either may be NULL. */
@@ -225,6 +236,27 @@ kvc_status kvc_decode_attention(kvc_cache* cache, int layer, const void* q, floa
  *     counters it relies on before its kernel runs, on `stream`. */
 kvc_status kvc_decode_attention_static_scratch(kvc_cache* cache, int layer, const void* q, float scale, float* out,
                                                void* stream);
+
+/* Masked prefill attention of layer `layer` on the tensor cores (Sec. 3.1: the modified causal
+ * mask holds for every token of a prompt; Manipulating Key-Value Memory: a long prefix may be run
+ * block by block).  For every sequence s with n_q[s] > 0 the queries are its last n_q[s] tokens;
+ * each attends, under the mask, to the stored rows of s -- exactly the rows a decode step at that
+ * token would see (the per-row rule is kvc_book_prefill_keys').
+ *   q:   device [sum n_q][H][d_head] in the cache dtype, sequence-major (sequence s's queries
+ *        consecutive, oldest first), NOT rotated: the kernel rotates each query at its token's
+ *        stored position when rotary_dim > 0, then rounds it to the cache dtype; 16-byte aligned.
+ *   n_q: host [b], 0 <= n_q[s] <= tokens of s.
+ *   out: device fp32 [sum n_q][H][d_head] = sum_j softmax_j(scale * <q, k_j>) v_j, 16-byte aligned.
+ *   scale: > 0.
+ * The queries' own K/V rows must be stored: append a block with kvc_append (every layer up to
+ * `layer` written), run the prefill of each layer, then free the spans the block closed with
+ * kvc_compress_spans -- the "for-loop over blocks" of Sec. 3.1.  Spans closed earlier may still be
+ * stored (their rows are masked), so a whole prompt can also be appended and run in one call.
+ * Errors: KVC_ERR_STATE when a query token is not stored (for example freed by
+ * kvc_append_free_closed) or its layer is not written; KVC_ERR_UNSUPPORTED under
+ * KVC_POLICY_LOCAL or when M * H * sum(capacity) >= 2^31 rows.  Asynchronous. */
+kvc_status kvc_prefill_attention(kvc_cache* cache, int layer, const void* q, const int32_t* n_q, float scale,
+                                 float* out, void* stream);
 
 /* Verification (synchronous: waits for `stream`): the history of `seq` and the mask for its next
  * query as in kvc_book_layout, with the stored rows read back from the device metadata

@@ -14,7 +14,7 @@ import numpy as np
 import synth
 from synth import workloads as wl
 
-from . import local_decode, masked_decode, tied_positions, POLICY_PAPER
+from . import local_decode, masked_decode, masked_prefill, tied_positions, POLICY_PAPER
 
 
 def history(w: wl.Workload, s: int, steps_done: int):
@@ -78,3 +78,25 @@ def expected_local_decode(w: wl.Workload, steps_done: int, layer: int, seqs, rat
         q_l.append(q_bits(w, layer, s, T - 1, heads))
     return local_decode(pos_l, K_l, V_l, np.stack(q_l), w.dtype, w.scale, ratio, rot=w.rotary_dim, base=w.rope_base,
                         n_threads=n_threads)
+
+
+def expected_prefill(w: wl.Workload, layer: int, seqs, end, n_q, heads=None, policy: int = POLICY_PAPER,
+                     n_threads: int = 0) -> np.ndarray:
+    """fp64 [sum n_q over seqs, n_heads, d]: masked prefill of `layer` for prompt tokens
+    [end[s] - n_q[s], end[s]) of each listed sequence, over its prompt history [0, end[s])."""
+    kinds_l, pos_l, K_l, V_l, Q_l, nq_l = [], [], [], [], [], []
+    for s in seqs:
+        T, n = int(end[s]), int(n_q[s])
+        kinds = np.asarray(w.prompt_kinds[s][:T], dtype=np.uint8)
+        K, V = kv_bits(w, layer, s, T, heads)
+        t = np.arange(T - n, T, dtype=np.int32)
+        Q = synth.fill_tokens_host(w.seed, w.dtype, synth.scale_for(w.q_sigma), synth.tag(synth.Q_TENSOR, layer), t,
+                                   np.full(n, s, np.int32), w.H, w.d)
+        kinds_l.append(kinds)
+        pos_l.append(tied_positions(kinds))
+        K_l.append(K)
+        V_l.append(V)
+        Q_l.append(Q if heads is None else Q[:, heads])
+        nq_l.append(n)
+    return masked_prefill(kinds_l, pos_l, K_l, V_l, nq_l, np.concatenate(Q_l), w.dtype, w.scale, rot=w.rotary_dim,
+                          base=w.rope_base, policy=policy, n_threads=n_threads)

@@ -132,6 +132,17 @@ def kvc_book_lengths(book: int, b: int):
     return ln, at
 
 
+def kvc_book_prefill_keys(book: int, seq: int, n_q: int) -> np.ndarray:
+    """Per stored row of `seq`: (hid << 1) | is_cl, the masked-prefill bounds for its last n_q tokens."""
+    n = ctypes.c_int64()
+    rc = lib().kvc_book_prefill_keys(book, seq, n_q, None, 0, ctypes.byref(n))
+    if rc != 0 and n.value == 0:
+        _check(rc)
+    meta = np.empty(max(n.value, 1), np.int32)
+    _check(lib().kvc_book_prefill_keys(book, seq, n_q, meta.ctypes.data, n.value, ctypes.byref(n)))
+    return meta[:n.value].copy()
+
+
 def _layout_sizes(fn, *args):
     nf, ns = ctypes.c_int64(), ctypes.c_int64()
     rc = fn(*args, 0, None, None, None, ctypes.byref(nf), None, None, ctypes.byref(ns))
@@ -187,6 +198,9 @@ class Book:
 
     def pending_spans(self, seq: int):
         return kvc_book_pending_spans(self.handle, seq)
+
+    def prefill_keys(self, seq: int, n_q: int) -> np.ndarray:
+        return kvc_book_prefill_keys(self.handle, seq, n_q)
 
     def lengths(self):
         return kvc_book_lengths(self.handle, self.b)
@@ -269,6 +283,12 @@ def kvc_decode_attention_static_scratch(cache: int, layer: int, q, scale: float,
     """Decode whose split-K scratch is the library's static device array (no allocation anywhere)."""
     _check(lib().kvc_decode_attention_static_scratch(cache, layer, _ptr(q), float(scale), _ptr(out),
                                                      _stream_handle(stream)))
+
+
+def kvc_prefill_attention(cache: int, layer: int, q, n_q, scale: float, out, stream=None):
+    n_q = _np(n_q, np.int32)
+    _check(lib().kvc_prefill_attention(cache, layer, _ptr(q), n_q.ctypes.data, float(scale), _ptr(out),
+                                       _stream_handle(stream)))
 
 
 def kvc_masked_reference_layout(cache: int, seq: int, cap: int, stream=None):
@@ -375,6 +395,21 @@ class KVCache:
         _dev(out, "out", torch.float32, self.b * self.H * self.d)
         kvc_decode_attention(self.handle, layer, q, scale, out, stream)
         return out
+
+    def prefill_attention(self, layer: int, q, n_q, scale: float, out=None, stream=None):
+        """Masked prefill of the last n_q[s] tokens of every sequence s (q: [sum n_q, H, d_head])."""
+        import torch
+
+        n_tok = int(np.sum(n_q))
+        _dev(q, "q", self.torch_dtype, n_tok * self.H * self.d)
+        if out is None:
+            out = torch.empty(n_tok, self.H, self.d, dtype=torch.float32, device=q.device)
+        _dev(out, "out", torch.float32, n_tok * self.H * self.d)
+        kvc_prefill_attention(self.handle, layer, q, n_q, scale, out, stream)
+        return out
+
+    def prefill_keys(self, seq: int, n_q: int) -> np.ndarray:
+        return kvc_book_prefill_keys(lib().kvc_get_book(self.handle), seq, n_q)
 
     def masked_reference_layout(self, seq: int, stream=None):
         cap = _layout_sizes(lib().kvc_book_layout, lib().kvc_get_book(self.handle), seq)

@@ -46,6 +46,7 @@ SIGNATURES = [
     ("kvc_book_compress", c_int, [P, P, P, P, c_int]),
     ("kvc_book_pending_spans", c_int, [P, c_int, P, P, c_int64, P]),
     ("kvc_book_lengths", c_int, [P, P, P]),
+    ("kvc_book_prefill_keys", c_int, [P, c_int, c_int64, P, c_int64, P]),
     ("kvc_book_layout", c_int, [P, c_int, c_int64, P, P, P, P, P, P, P]),
     ("kvc_required_bytes", c_int, [P, P, P, P, P]),
     ("kvc_create", c_int, [P, P]),
@@ -56,6 +57,7 @@ SIGNATURES = [
     ("kvc_compress_spans", c_int, [P, P, P, P, c_int, P]),
     ("kvc_decode_attention", c_int, [P, c_int, P, c_float, P, P]),
     ("kvc_decode_attention_static_scratch", c_int, [P, c_int, P, c_float, P, P]),
+    ("kvc_prefill_attention", c_int, [P, c_int, P, P, c_float, P, P]),
     ("kvc_masked_reference_layout", c_int, [P, c_int, c_int64, P, P, P, P, P, P, P, P]),
     ("kvc_device_status", c_int, [P, P, P]),
     ("kvc_launch_count", c_int64, [P]),

@@ -12,8 +12,8 @@ OUT = os.path.join(HERE, "_build")
 SO = os.path.join(OUT, "libkvc.so")
 INCLUDE = os.path.join(ROOT, "include")
 GENCODE = "arch=compute_103a,code=sm_103a"
-SOURCES = ["kvc.cpp", "book.cpp", "kernels.cu"]
-HEADERS = [os.path.join(CSRC, h) for h in ("book.hpp", "kernels.hpp")] + [os.path.join(INCLUDE, "kvc.h")]
+SOURCES = ["kvc.cpp", "book.cpp", "kernels.cu", "prefill.cu"]
+HEADERS = [os.path.join(CSRC, h) for h in ("book.hpp", "kernels.hpp", "device_common.cuh")] + [os.path.join(INCLUDE, "kvc.h")]
 
 
 def _flags(verbose_ptx: bool = False):

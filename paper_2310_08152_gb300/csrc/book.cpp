@@ -355,6 +355,53 @@ bool Book::decode_view(int s, DecodeView& v, std::string& err) const {
   return true;
 }
 
+bool Book::prefill_keys(int s, int64_t n_q, std::vector<int32_t>& meta, std::string& err) const {
+  const Seq& q = seqs_[s];
+  const int64_t T = (int64_t)q.kind.size();
+  char buf[256];
+  meta.clear();
+  if (policy_ == POLICY_LOCAL) {
+    err = "masked prefill is not defined for the local-attention cache";
+    return false;
+  }
+  if (n_q < 0 || n_q > T) {
+    std::snprintf(buf, sizeof buf, "sequence %d: n_q = %lld outside [0, %lld]", s, (long long)n_q, (long long)T);
+    err = buf;
+    return false;
+  }
+  if (n_q == 0) return true;
+  if (q.stored >= kPrefillNever) {
+    std::snprintf(buf, sizeof buf, "sequence %d: %lld stored rows exceed the prefill limit", s, (long long)q.stored);
+    err = buf;
+    return false;
+  }
+  // the queries are the last n_q tokens and must all be stored rows (the tail of the stored rows)
+  if (q.stored < n_q || stored_index(s, T - n_q) != q.stored - n_q) {
+    std::snprintf(buf, sizeof buf,
+                  "sequence %d: the last %lld tokens are not all stored (append them without freeing and "
+                  "compress after the prefill)",
+                  s, (long long)n_q);
+    err = buf;
+    return false;
+  }
+  meta.assign((size_t)q.stored, kPrefillNever << 1);
+  for (int64_t j = 0; j < T; ++j) {
+    if (q.kind[j] != CL) continue;
+    const int64_t i = stored_index(s, j);
+    if (i < 0) continue;
+    meta[i] = policy_ == POLICY_PAPER ? (int32_t)((i << 1) | 1) : (int32_t)((kPrefillNever << 1) | 1);
+  }
+  for (const Span& sp : q.spans) {
+    if (sp.freed || sp.cr < 0) continue;
+    const int64_t hid = stored_index(s, sp.cr);
+    for (int64_t j = sp.cl + 1; j < sp.cr; ++j) {
+      const int64_t i = stored_index(s, j);
+      if (i >= 0) meta[i] = (int32_t)((hid << 1) | (meta[i] & 1));
+    }
+  }
+  return true;
+}
+
 void Book::pending_spans(int s, std::vector<std::pair<int64_t, int64_t>>& out) const {
   out.clear();
   for (const Span& sp : seqs_[s].spans)

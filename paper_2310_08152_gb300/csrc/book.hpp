@@ -79,6 +79,15 @@ class Book {
   // are not one contiguous run of stored rows.
   bool decode_view(int s, DecodeView& v, std::string& err) const;
 
+  // Masked prefill of the last n_q history tokens of sequence s over its stored rows (Sec. 3.1).
+  // meta[i] = (hid << 1) | is_cl for stored row i: row i is visible to the query at stored row iq
+  // exactly when i <= iq <= hid, except that a <CL> query (is_cl of its own row) sees only itself.
+  // hid is the stored row of the <CR> closing a span that encloses row i, i itself for a <CL> row
+  // under the paper policy, else kPrefillNever.  False (with `err`) when the policy has no prefill
+  // or the queries are not the last n_q stored rows.
+  static constexpr int32_t kPrefillNever = 0x3FFFFFFF;
+  bool prefill_keys(int s, int64_t n_q, std::vector<int32_t>& meta, std::string& err) const;
+
   void pending_spans(int s, std::vector<std::pair<int64_t, int64_t>>& out) const;
   // history index -> stored row (or -1 when freed)
   int64_t stored_index(int s, int64_t j) const;

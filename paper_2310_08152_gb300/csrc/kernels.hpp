@@ -94,6 +94,45 @@ struct DecodePlan {
 cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a,
                           int num_sms, cudaStream_t stream, int* grid, DecodePlan* plan);
 
+// ---------------------------------------------------------------------------------------------
+// Masked prefill attention (prefill.cu)
+// ---------------------------------------------------------------------------------------------
+// Per sequence: stored rows [0, len); the queries are stored rows [q0, len), the first of them is
+// token qtok of the q / out arrays; the per-row mask bounds start at meta[moff].
+struct PState {
+  int32_t len, q0, qtok, moff;
+};
+
+struct PrefillArgs {
+  int layer, H, b, rot;
+  int64_t C;
+  const PState* ps;        // [b]
+  const int32_t* Pq;       // [b+1] prefix sums of query tiles (128 queries each)
+  const int32_t* meta;     // per stored row: (hid << 1) | is_cl
+  const uint16_t* q;       // [sum n_q][H][D]
+  float* out;              // [sum n_q][H][D]
+  float c2;                // scale * log2(e)
+  const int32_t* pos;      // [C] stored-row positions
+  const int64_t* off;      // [b]
+  const int64_t* seq_row0; // [b]
+  const int32_t* cap;      // [b]
+  const float2* rope_g;    // [rot/2]
+  int* status;
+  unsigned long long wait_limit_ns;
+};
+
+// Encoded 2-D TMA descriptors of the K and V planes ([M*H*C rows][D], swizzled column subtiles).
+struct alignas(64) PrefillMaps {
+  unsigned char k[128];
+  unsigned char v[128];
+  bool ready = false;
+};
+
+cudaError_t encode_prefill_maps(const Geometry& g, const Buffers& buf, PrefillMaps* maps);
+// grid = H * Pq[b] CTAs
+cudaError_t launch_prefill(const Geometry& g, const PrefillMaps& maps, const PrefillArgs& a, int64_t grid,
+                           cudaStream_t stream);
+
 // One warp waits on an mbarrier phase that never completes, with the limit given; the bounded wait
 // gives up and sets STATUS_TIMEOUT in *status.  Exercises the kernels' timeout reporting.
 cudaError_t launch_bounded_wait_check(int* status, unsigned long long limit_ns, cudaStream_t stream);

@@ -58,6 +58,10 @@ struct WsLayout {
   size_t src_map = 0;    // int32 [C]: source row of each destination row of a compaction
   size_t counters = 0;   // int32 [b*H]
   size_t partials = 0;   // float [(kMaxDecodeWorkers + b*H) * (D + 4)]
+  size_t pre = 0;        // prefill plan: [PState b][int32 Pq b+1][int32 meta C]
+  size_t pre_Pq = 0;     // offsets inside the prefill plan
+  size_t pre_meta = 0;
+  size_t pre_bytes = 0;
   size_t total = 0;
 };
 
@@ -83,6 +87,10 @@ WsLayout ws_layout(int b, int H, int D, int rot, int64_t C) {
   L.src_map = take(4 * (size_t)C);
   L.counters = take(4 * (size_t)b * H);
   L.partials = take(4 * (size_t)(kvc::kMaxDecodeWorkers + (int64_t)b * H) * (size_t)(D + 4));
+  L.pre_Pq = align_up(sizeof(kvc::PState) * (size_t)b, 16);
+  L.pre_meta = align_up(L.pre_Pq + 4 * (size_t)(b + 1), 16);
+  L.pre_bytes = L.pre_meta + 4 * (size_t)C;
+  L.pre = take(L.pre_bytes);
   L.total = o;
   return L;
 }
@@ -214,6 +222,12 @@ struct kvc_cache {
   // the last kernel this cache launched was a decode (it writes no K/V rows)
   bool last_was_decode = false;
   kvc::DecodePlan last_plan{-1, 0, 0, 0};
+  // book changes (appends, compactions); the prefill plan is rebuilt when it moved on
+  uint64_t version = 0;
+  uint64_t pre_version = UINT64_MAX;
+  std::vector<int32_t> pre_nq;
+  int64_t pre_tiles = 0;
+  kvc::PrefillMaps maps;
 
   kvc_cache(const kvc_config& c, int64_t C_)
       : cfg(c), C(C_), bk(c.b, (kvc::Policy)c.policy, c.seq_capacity, (double)c.local_ratio) {
@@ -269,7 +283,7 @@ struct kvc_cache {
     }
     e = cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
-    e = ring.init(2 * ws.dyn_bytes + 2 * ws.st_rope + 65536);
+    e = ring.init(2 * ws.dyn_bytes + ws.pre_bytes + 2 * ws.st_rope + 65536);
     if (e != cudaSuccess) return cuda_fail(e, "cudaHostAlloc (staging ring)");
     // static tables
     const int b = cfg.b, half = std::max(1, cfg.rotary_dim / 2);
@@ -305,6 +319,7 @@ struct kvc_cache {
 
   // Fill the decode state + prefix at the head of a dyn image.
   void fill_state(unsigned char* img) {
+    ++version;
     kvc::DState* ds = reinterpret_cast<kvc::DState*>(img);
     int64_t* P = reinterpret_cast<int64_t*>(img + ws.dyn_P);
     decode_ok = true;
@@ -471,6 +486,23 @@ kvc_status kvc_book_pending_spans(const kvc_book* book, int seq, int64_t* cl, in
     if (cl) cl[i] = v[i].first;
     if (cr) cr[i] = v[i].second;
   }
+  return ok();
+}
+
+kvc_status kvc_book_prefill_keys(const kvc_book* book, int seq, int64_t n_q, int32_t* meta, int64_t max,
+                                 int64_t* n) {
+  if (!book || !n) return fail(KVC_ERR_INVALID_ARG, "book/n is NULL");
+  if (seq < 0 || seq >= book->book.b()) return fail(KVC_ERR_INVALID_ARG, "seq %d out of range", seq);
+  if (book->book.policy() == kvc::POLICY_LOCAL)
+    return fail(KVC_ERR_UNSUPPORTED, "masked prefill is not defined for the local-attention cache");
+  std::vector<int32_t> m;
+  std::string err;
+  if (!book->book.prefill_keys(seq, n_q, m, err)) return fail(KVC_ERR_STATE, "%s", err.c_str());
+  *n = (int64_t)m.size();
+  if ((int64_t)m.size() > max) return fail(KVC_ERR_INVALID_ARG, "meta holds %lld entries, %lld needed", (long long)max,
+                                           (long long)m.size());
+  if (!m.empty() && !meta) return fail(KVC_ERR_INVALID_ARG, "meta is NULL");
+  std::memcpy(meta, m.data(), 4 * m.size());
   return ok();
 }
 
@@ -792,6 +824,98 @@ kvc_status kvc_decode_attention_static_scratch(kvc_cache* c, int layer, const vo
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel (static scratch)");
   c->launches += grid > 0 ? 1 : 0;
   c->last_was_decode = true;
+  return ok();
+}
+
+kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const int32_t* n_q, float scale, float* out,
+                                 void* stream_) {
+  if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  const int b = c->cfg.b, H = c->cfg.H, D = c->cfg.d_head;
+  if (layer < 0 || layer >= c->cfg.M) return fail(KVC_ERR_INVALID_ARG, "layer %d out of range", layer);
+  if (!q || !out || !n_q) return fail(KVC_ERR_INVALID_ARG, "q/out/n_q are NULL");
+  if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out)) & 15)
+    return fail(KVC_ERR_INVALID_ARG, "q and out must be 16-byte aligned");
+  if (!(scale > 0.0f) || !std::isfinite(scale)) return fail(KVC_ERR_INVALID_ARG, "scale must be positive and finite");
+  if (c->cfg.policy == KVC_POLICY_LOCAL)
+    return fail(KVC_ERR_UNSUPPORTED, "masked prefill is not defined for the local-attention cache");
+  if ((int64_t)c->cfg.M * H * c->C >= ((int64_t)1 << 31))
+    return fail(KVC_ERR_UNSUPPORTED, "M*H*sum(capacity) rows exceed the 2^31 rows a tensor-map coordinate reaches");
+  if (layer >= c->layers_done) return fail(KVC_ERR_STATE, "layer %d of the last tokens is not written yet", layer);
+  for (int s = 0; s < b; ++s)
+    if (n_q[s] < 0 || n_q[s] > c->bk.book.history(s))
+      return fail(KVC_ERR_INVALID_ARG, "n_q[%d] = %d outside [0, %lld]", s, n_q[s],
+                  (long long)c->bk.book.history(s));
+  if (!c->cuda_ready) return fail(KVC_ERR_STATE, "nothing appended yet");
+  kvc_status st = c->ensure_cuda(stream);
+  if (st != KVC_OK) return st;
+  cudaError_t e;
+  if (!c->maps.ready) {
+    e = kvc::encode_prefill_maps(c->geom(), c->bufs(), &c->maps);
+    if (e != cudaSuccess) return cuda_fail(e, "cuTensorMapEncodeTiled (K/V planes)");
+  }
+  const bool same = c->pre_version == c->version && std::equal(c->pre_nq.begin(), c->pre_nq.end(), n_q) &&
+                    (int)c->pre_nq.size() == b;
+  if (!same) {
+    // per-sequence state, tile prefix and per-row mask bounds
+    std::vector<std::vector<int32_t>> metas(b);
+    size_t n_meta = 0;
+    for (int s = 0; s < b; ++s) {
+      std::string err;
+      if (!c->bk.book.prefill_keys(s, n_q[s], metas[s], err)) return fail(KVC_ERR_STATE, "%s", err.c_str());
+      n_meta += metas[s].size();
+    }
+    const size_t bytes = c->ws.pre_meta + 4 * n_meta;
+    unsigned char* img = c->ring.reserve(bytes, &e);
+    if (!img) return e != cudaSuccess ? cuda_fail(e, "staging") : fail(KVC_ERR_INVALID_ARG, "prefill plan exceeds ring");
+    kvc::PState* ps = reinterpret_cast<kvc::PState*>(img);
+    int32_t* Pq = reinterpret_cast<int32_t*>(img + c->ws.pre_Pq);
+    int32_t* meta = reinterpret_cast<int32_t*>(img + c->ws.pre_meta);
+    int64_t qtok = 0, moff = 0;
+    Pq[0] = 0;
+    for (int s = 0; s < b; ++s) {
+      const int64_t len = c->bk.book.stored(s);
+      ps[s].len = (int32_t)len;
+      ps[s].q0 = (int32_t)(len - n_q[s]);
+      ps[s].qtok = (int32_t)qtok;
+      ps[s].moff = (int32_t)moff;
+      std::memcpy(meta + moff, metas[s].data(), 4 * metas[s].size());
+      moff += (int64_t)metas[s].size();
+      qtok += n_q[s];
+      Pq[s + 1] = Pq[s] + (n_q[s] + 127) / 128;
+    }
+    e = c->ring.commit(c->wsp(c->ws.pre), bytes, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "upload prefill plan");
+    c->pre_version = c->version;
+    c->pre_nq.assign(n_q, n_q + b);
+    c->pre_tiles = Pq[b];
+  }
+  if (c->pre_tiles == 0) return ok();
+  kvc::PrefillArgs a;
+  a.layer = layer;
+  a.H = H;
+  a.b = b;
+  a.rot = c->cfg.rotary_dim;
+  a.C = c->C;
+  a.ps = reinterpret_cast<const kvc::PState*>(c->wsp(c->ws.pre));
+  a.Pq = reinterpret_cast<const int32_t*>(c->wsp(c->ws.pre + c->ws.pre_Pq));
+  a.meta = reinterpret_cast<const int32_t*>(c->wsp(c->ws.pre + c->ws.pre_meta));
+  a.q = static_cast<const uint16_t*>(q);
+  a.out = out;
+  a.c2 = (float)((double)scale * 1.4426950408889634);
+  a.pos = c->cfg.pos_base;
+  const kvc::Static sta = c->stat();
+  a.off = sta.off;
+  a.seq_row0 = sta.seq_row0;
+  a.cap = sta.cap;
+  a.rope_g = sta.rope_g;
+  a.status = c->bufs().status;
+  a.wait_limit_ns = 2000000000ull;
+  (void)D;
+  e = kvc::launch_prefill(c->geom(), c->maps, a, (int64_t)H * c->pre_tiles, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "prefill kernel");
+  c->launches += 1;
+  c->last_was_decode = false;
   return ok();
 }
 

@@ -327,3 +327,74 @@ def test_local_book_capacity_is_the_window():
     assert book.lengths()[0][0] == 10
     book.append([1], [NORMAL])  # x_20 sees (10, 20]: still 10
     assert _err(book.append, [2], [NORMAL, NORMAL]) == 3  # x_22 would see (11, 22]: 11 rows
+
+
+def _wellformed(n):
+    import itertools
+    for seq in itertools.product((NORMAL, CL, CR), repeat=n):
+        open_ = False
+        ok = True
+        for k in seq:
+            if (k == CL and open_) or (k == CR and not open_):
+                ok = False
+                break
+            if k != NORMAL:
+                open_ = k == CL
+        if ok:
+            yield np.array(seq, np.uint8)
+
+
+def _prefill_visible(meta, iq):
+    """The documented prefill rule: row i is visible to the query at stored row iq iff
+    i <= iq <= hid(i), and a <CL> query (its own is_cl bit) sees only itself."""
+    hid = meta >> 1
+    i = np.arange(meta.size)
+    vis = (i <= iq) & (iq <= hid)
+    if meta[iq] & 1:
+        vis = i == iq
+    return vis
+
+
+@pytest.mark.parametrize("policy", [kvc.POLICY_PAPER, kvc.POLICY_KEEP_CL])
+def test_book_prefill_mask_bounds_match_oracle_bruteforce(policy):
+    """Every well-formed history of up to 7 tokens, split into a first part (appended, its closed
+    spans freed) and a prefill block: the per-row bounds give, for every query of the block, exactly
+    the oracle's visible set mapped onto the stored rows (Sec. 3.1 mask)."""
+    n_checked = 0
+    for n in range(1, 8):
+        for kinds in _wellformed(n):
+            for k in range(n):  # block = tokens [k, n)
+                book = kvc.Book(1, [n], policy)
+                if k:
+                    book.append([k], kinds[:k])
+                    spans = book.pending_spans(0)
+                    if spans:
+                        book.compress([0] * len(spans), [a for a, _ in spans], [c for _, c in spans])
+                book.append([n - k], kinds[k:])
+                meta = book.prefill_keys(0, n - k)
+                rows = book.layout(0)["stored_orig"]
+                assert meta.size == rows.size
+                for t in range(k, n):
+                    iq = int(np.nonzero(rows == t)[0][0])
+                    assert iq == rows.size - (n - t)  # the queries are the last stored rows
+                    vis_hist = orc.visible(kinds[:t + 1], t, policy)
+                    expect = np.zeros(rows.size, bool)
+                    for r, j in enumerate(rows):
+                        expect[r] = j <= t and vis_hist[j]
+                    assert np.array_equal(_prefill_visible(meta, iq), expect), (kinds, k, t)
+                    # nothing the query may see was freed
+                    assert set(np.nonzero(vis_hist)[0]) <= set(rows.tolist())
+                    n_checked += 1
+    assert n_checked > 5000
+
+
+def test_book_prefill_keys_errors():
+    book = kvc.Book(1, [16])
+    book.append([6], [NORMAL, CL, NORMAL, CR, NORMAL, NORMAL], free_closed=True)  # rows 1..2 freed
+    assert _err(book.prefill_keys, 0, 5) == 5   # token 1 is not stored
+    assert _err(book.prefill_keys, 0, 7) == 5   # more queries than tokens
+    assert book.prefill_keys(0, 3).size == 4    # tokens 3..5 are the last stored rows
+    assert book.prefill_keys(0, 0).size == 0
+    local = kvc.Book(1, [16], kvc.POLICY_LOCAL, local_ratio=0.5)
+    local.append([3], [NORMAL] * 3)
+    assert _err(local.prefill_keys, 0, 1) == 2
