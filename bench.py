@@ -48,6 +48,10 @@ def parse():
                     help="largest batch under a KV-memory cap per compression ratio, and its throughput")
     ap.add_argument("--caps", default="12,24,180", help="KV-memory caps in GB for --capacity-sweep")
     ap.add_argument("--ratios", default="0,0.5,0.8,0.9", help="compression ratios for --capacity-sweep")
+    ap.add_argument("--prefill-only", action="store_true",
+                    help="only time the masked prefill of the workload's prompt (one JSON line per mode)")
+    ap.add_argument("--prefill-block", type=int, default=-1,
+                    help="with --prefill-only: block size (0 = one go; default: both 0 and 512)")
     return ap.parse_args()
 
 
@@ -59,6 +63,18 @@ def measured_hbm_peak():
         return float(j["hbm_gbs"]), "measured"
     except Exception:
         return FALLBACK_HBM_GBS, "fallback"
+
+
+def measured_tensor_peak():
+    """Dense 16-bit tensor-core TFLOP/s measured by a cuBLAS bf16 GEMM (burst); f16 runs at the same
+    dense rate on these tensor cores."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            j = json.load(f)
+        return float(j["bf16_tflops"]), "measured (bf16 GEMM burst; same dense rate for f16)"
+    except Exception:
+        return 1900.0, "fallback"
 
 
 def kernel_source_hash() -> str:
@@ -360,6 +376,75 @@ def time_prompt_write_time_freeing(w, steps_total, dev):
             "rows_written_per_stream": stored, "rows_in_prompt_per_stream": int(w.prompt_len.sum())}
 
 
+def prefill_work(w, block: int):
+    """FLOPs of one layer's masked prefill over the prompt, summed over sequences and heads:
+    (algorithmic) 4 d per visible (query, key) pair -- q.k and p.v over exactly the rows the mask
+    leaves (Sec. 3.1) -- and (executed) 4 d x 128 x 128 per key tile the kernel runs.  The visible
+    counts follow the per-row bounds of the library's host book: query iq sees rows i <= iq with
+    hid(i) >= iq, a <CL> query only itself."""
+    import paper_2310_08152_gb300 as kvc
+
+    L = w.prompt_len
+    book = kvc.Book(w.b, L + 1)
+    start = np.zeros(w.b, np.int64)
+    pairs = tiles = 0
+    while (start < L).any():
+        n = L - start if block <= 0 else np.minimum(L - start, block)
+        kinds = np.concatenate([w.prompt_kinds[s][start[s]:start[s] + n[s]] for s in range(w.b)]).astype(np.uint8)
+        book.append(n.astype(np.int32), kinds)
+        for s in range(w.b):
+            if n[s] == 0:
+                continue
+            meta = book.prefill_keys(s, int(n[s]))
+            hid, cl = meta >> 1, meta & 1
+            ln = meta.size
+            q0 = ln - int(n[s])
+            iq = np.arange(q0, ln)
+            cnt = (iq + 1) - np.searchsorted(np.sort(hid), iq, side="left")
+            pairs += int(np.where(cl[iq] == 1, 1, cnt).sum())
+            for qt in range((int(n[s]) + 127) // 128):
+                tiles += (min(q0 + 128 * (qt + 1), ln) + 127) // 128
+        seq, cl_, cr_ = [], [], []
+        for s in range(w.b):
+            for a, c in book.pending_spans(s):
+                seq.append(s)
+                cl_.append(a)
+                cr_.append(c)
+        if seq:
+            book.compress(seq, cl_, cr_)
+        start = start + n
+    return 4 * w.d * pairs * w.H, 4 * w.d * 128 * 128 * tiles * w.H
+
+
+def time_prompt_prefill(w, steps_total, dev, block: int):
+    """Prompt ingestion with masked prefill attention of every layer (tensor cores), one go
+    (block 0) or block by block with the closed spans freed in between; reports the prefill kernel's
+    TFLOP/s (algorithmic: visible pairs only) against the measured dense 16-bit peak."""
+    import torch
+
+    import harness
+
+    run = harness.Runner(w, steps_total, device=dev)
+    ev = []
+    run.prefill_prompt(block=block, events=ev)
+    torch.cuda.synchronize()
+    ms = [a.elapsed_time(b) for a, b in ev]
+    status = run.cache.device_status()
+    del run
+    torch.cuda.empty_cache()
+    alg, executed = prefill_work(w, block)
+    total_s = sum(ms) / 1e3
+    n_blocks = max(1, len(ms) // w.M)
+    peak, kind = measured_tensor_peak()
+    achieved = alg * w.M / total_s / 1e12
+    return {"kernel": "prefill_kernel (tcgen05.mma, TMEM accumulators, TMA-swizzled K/V)",
+            "mode": "one go" if block <= 0 else f"blocks of {block} tokens", "launches": len(ms),
+            "ms_total": sum(ms), "ms_per_layer": sum(ms) / w.M, "blocks": n_blocks,
+            "tflop_per_layer_algorithmic": alg / 1e12, "tflop_per_layer_executed": executed / 1e12,
+            "achieved": achieved, "executed_tflops": executed * w.M / total_s / 1e12, "peak": peak,
+            "unit": "TFLOP/s", "frac": achieved / peak, "peak_kind": kind, "device_status": status}
+
+
 def run_capacity_sweep(args):
     """Largest batch whose compressed KV cache fits a memory cap, and its decode-step throughput, for
     several compression ratios: a synthetic restatement of the paper's throughput-vs-VRAM experiment
@@ -431,6 +516,7 @@ def run_kvc(args, w):
     torch.cuda.synchronize()
     compaction["prompt_append_ms"] = sum(a.elapsed_time(b) for a, b in append_ev)
     prompt_free = time_prompt_write_time_freeing(w, steps_total, dev)
+    prefill = [time_prompt_prefill(w, steps_total, dev, blk) for blk in (0, 512)]
     inputs = [run.make_step_inputs(g) for g in range(steps_total)]
     out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device=dev)
     torch.cuda.synchronize()
@@ -513,6 +599,7 @@ def run_kvc(args, w):
             "decode_share_of_step": dec_total_s / elapsed,
             "compaction": compaction,
             "prompt_write_time_freeing": prompt_free,
+            "prefill": prefill,
             "gpu_launches": launches,
             "device_status": status,
             "clocks": clk,
@@ -587,6 +674,17 @@ def main():
         import dataclasses
 
         w = dataclasses.replace(w, M=args.layers, name=f"{w.name}-M{args.layers}")
+    if args.prefill_only:
+        import torch
+
+        torch.cuda.set_device(0)
+        dev = torch.device("cuda", 0)
+        blocks = (0, 512) if args.prefill_block < 0 else (args.prefill_block,)
+        for blk in blocks:
+            r = time_prompt_prefill(w, 1, dev, blk)
+            r["workload"] = w.name
+            print(json.dumps(r), flush=True)
+        return
     if args.impl == "reference":
         run_reference(args, w)
     else:
