@@ -33,7 +33,6 @@ namespace {
 
 constexpr int kPfRows = 128;     // queries per tile (MMA M) and keys per tile (QK^T N, PV K)
 constexpr int kPfThreads = 192;  // producer warp, MMA warp, 4 softmax warps
-constexpr int kPfNever = 0x3FFFFFFF;
 
 // Shared-memory geometry for head dimension D.  Q, K and V tiles are [128 rows][D] split into
 // column subtiles of SW bytes per row, the widest swizzle (128 / 64 / 32 bytes) that divides a row;
@@ -210,8 +209,12 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   extern __shared__ uint8_t pf_smem_raw[];
   __shared__ uint64_t full_bar[NST], empty_bar[NST], s_full[2], s_free[2];
   __shared__ uint64_t q_full, p_full, pv_done, drain;
-  __shared__ int32_t kmeta[NST][kPfRows];
-  __shared__ int32_t kmin[NST];
+  // Per stage, the tile's keys against this CTA's query tile [qr0, qr_end): khid has bit c set when
+  // key c's bound holds for every query of the tile (hid >= qr_end - 1); klist holds the keys whose
+  // bound falls inside it (qr0 <= hid < qr_end - 1: a span closing among the queries), kn of them.
+  __shared__ uint4 khid[NST];
+  __shared__ int2 klist[NST][kPfRows];
+  __shared__ int32_t kn[NST];
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
 
@@ -287,18 +290,26 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         }
       }
       ++issued;
-      // per-key mask bounds of the tile: (hid << 1) | is_cl; rows past the stored ones are invisible
-      int mn = kPfNever;
+      // per-key mask bounds of the tile ((hid << 1) | is_cl; rows past the stored ones: invisible)
+      // sorted into the classes above; the causal part (i <= iq) is left to each query
+      uint32_t ok_w[4];
+      int n_part = 0;
 #pragma unroll
-      for (int c = lane; c < kPfRows; c += 32) {
+      for (int w4 = 0; w4 < 4; ++w4) {
+        const int c = lane + 32 * w4;
         const int i = kPfRows * j + c;
-        const int v = i < ps.len ? a.meta[ps.moff + i] : -2;
-        kmeta[st][c] = v;
-        mn = min(mn, v >> 1);
+        const int hid = (i < ps.len ? a.meta[ps.moff + i] : -2) >> 1;
+        ok_w[w4] = __ballot_sync(0xFFFFFFFFu, hid >= qr_end - 1);
+        const bool part = hid >= qr0 && hid < qr_end - 1;
+        const uint32_t pb = __ballot_sync(0xFFFFFFFFu, part);
+        if (part) klist[st][n_part + __popc(pb & ((1u << lane) - 1u))] = make_int2(c, hid);
+        n_part += __popc(pb);
       }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) mn = min(mn, __shfl_xor_sync(0xFFFFFFFFu, mn, o));
-      if (lane == 0) kmin[st] = mn;
+      if (lane == 0) {
+        khid[st] = make_uint4(ok_w[0], ok_w[1], ok_w[2], ok_w[3]);
+        kn[st] = n_part;
+      }
+      __syncwarp();
       mbar_arrive(&full_bar[st]);
     }
     if (!ok && lane == 0) {
@@ -414,31 +425,71 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       tc_fence_before();
       mbar_arrive(&s_free[sb]);
       const int kb = kPfRows * j;
-      const bool fast = (kb + kPfRows - 1 <= iq) && (kmin[st] >= iq) && !cl_q;
-      if (!fast) {
-#pragma unroll
-        for (int c = 0; c < kPfRows; ++c) {
-          const int mv = kmeta[st][c];
-          const int i = kb + c;
-          const bool vis = (i <= iq) && ((mv >> 1) >= iq) && (!cl_q || i == iq);
-          sv[c] = vis ? sv[c] : -INFINITY;
+      // visibility of the tile's keys to this query as four 32-bit words: the causal prefix
+      // (key row <= iq) and the tile-wide bound words, plus the listed keys whose bound admits iq; a
+      // <CL> query sees only its own row
+      const int t = iq - kb;  // last visible column
+      uint32_t v0, v1, v2, v3;
+      {
+        auto prefix = [t](int w) -> uint32_t {
+          const int n = t - 32 * w + 1;  // columns of word w at or before t
+          return n <= 0 ? 0u : n >= 32 ? 0xFFFFFFFFu : (1u << n) - 1u;
+        };
+        if (cl_q) {
+          auto one = [t](int w) -> uint32_t { return (t >> 5) == w ? 1u << (t & 31) : 0u; };
+          v0 = one(0), v1 = one(1), v2 = one(2), v3 = one(3);
+        } else {
+          const uint4 hw = khid[st];
+          v0 = hw.x, v1 = hw.y, v2 = hw.z, v3 = hw.w;
+          const int np = kn[st];
+          for (int e = 0; e < np; ++e) {
+            const int2 ent = klist[st][e];
+            if (ent.y >= iq) {
+              const uint32_t bit = 1u << (ent.x & 31);
+              const int w = ent.x >> 5;
+              v0 |= w == 0 ? bit : 0u;
+              v1 |= w == 1 ? bit : 0u;
+              v2 |= w == 2 ? bit : 0u;
+              v3 |= w == 3 ? bit : 0u;
+            }
+          }
+          v0 &= prefix(0), v1 &= prefix(1), v2 &= prefix(2), v3 &= prefix(3);
         }
       }
-      float mx = sv[0];
+      if ((v0 & v1 & v2 & v3) != 0xFFFFFFFFu) {
 #pragma unroll
-      for (int c = 1; c < kPfRows; ++c) mx = fmaxf(mx, sv[c]);
-      const float m_new = fmaxf(m, mx * c2);
+        for (int e = 0; e < 32; ++e) {
+          sv[e] = (v0 >> e) & 1u ? sv[e] : -INFINITY;
+          sv[32 + e] = (v1 >> e) & 1u ? sv[32 + e] : -INFINITY;
+          sv[64 + e] = (v2 >> e) & 1u ? sv[64 + e] : -INFINITY;
+          sv[96 + e] = (v3 >> e) & 1u ? sv[96 + e] : -INFINITY;
+        }
+      }
+      // row max: a tree over 8 partial maxima keeps the dependency chains short
+      float mx8[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) mx8[u] = sv[u];
+#pragma unroll
+      for (int c = 8; c < kPfRows; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], sv[c]);
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      // Reference maximum: moved only when the row maximum grows by more than 2^8 (log2 units), so O
+      // is rescaled rarely; P stays below 2^8 and its scale cancels exactly in O / l.
+      const float cand = mx * c2;
+      const bool move = cand > m + 8.f;
+      const float m_new = move ? cand : m;
       const float ref = m_new == -INFINITY ? 0.f : m_new;
       uint32_t pk[kPfRows / 2];
-      float rs = 0.f;
+      float rs8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int c = 0; c < kPfRows; c += 2) {
         const float p0 = ex2(fmaf(sv[c], c2, -ref));
         const float p1 = ex2(fmaf(sv[c + 1], c2, -ref));
-        rs += p0 + p1;
+        rs8[(c >> 1) & 7] += p0 + p1;
         pk[c / 2] = Pack16<T>::two(p0, p1);
       }
-      const float alpha = m == -INFINITY ? 0.f : ex2(m - ref);
+      const float rs = ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
+      const float alpha = !move ? 1.f : (m == -INFINITY ? 0.f : ex2(m - ref));
       l = l * alpha + rs;
       if (j >= 1) {
         // PV of the previous tile is complete: O may be rescaled and the P tile rewritten
