@@ -108,8 +108,12 @@ struct PrefillArgs {
   int64_t C;
   const PState* ps;        // [b]
   const int32_t* Pq;       // [b+1] prefix sums of query tiles (128 queries each)
+  int64_t n_items;         // H * Pq[b]: (query tile, head) work items
+  const int32_t* cta_items; // [n_ctas + 1]: CTA c takes items [cta_items[c], cta_items[c+1])
+  int n_ctas;              // persistent grid size
   const int32_t* meta;     // per stored row: (hid << 1) | is_cl
   const uint16_t* q;       // [sum n_q][H][D]
+  const uint16_t* v;       // cache V planes (a <CL> query's output is its own value row)
   float* out;              // [sum n_q][H][D]
   float c2;                // scale * log2(e)
   const int32_t* pos;      // [C] stored-row positions
@@ -129,9 +133,12 @@ struct alignas(64) PrefillMaps {
 };
 
 cudaError_t encode_prefill_maps(const Geometry& g, const Buffers& buf, PrefillMaps* maps);
-// grid = H * Pq[b] CTAs
-cudaError_t launch_prefill(const Geometry& g, const PrefillMaps& maps, const PrefillArgs& a, int64_t grid,
-                           cudaStream_t stream);
+// Most CTAs of the persistent prefill grid (sizes its work-range table).
+constexpr int kMaxPrefillCtas = 1024;
+// CTAs of the prefill kernel that fit on one SM for head dimension D (sizes the persistent grid).
+int prefill_ctas_per_sm(int D);
+// A persistent grid of a.n_ctas CTAs walks the a.n_items work items.
+cudaError_t launch_prefill(const Geometry& g, const PrefillMaps& maps, const PrefillArgs& a, cudaStream_t stream);
 
 // One warp waits on an mbarrier phase that never completes, with the limit given; the bounded wait
 // gives up and sets STATUS_TIMEOUT in *status.  Exercises the kernels' timeout reporting.

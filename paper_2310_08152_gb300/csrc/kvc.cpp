@@ -60,6 +60,7 @@ struct WsLayout {
   size_t partials = 0;   // float [(kMaxDecodeWorkers + b*H) * (D + 4)]
   size_t pre = 0;        // prefill plan: [PState b][int32 Pq b+1][int32 meta C]
   size_t pre_Pq = 0;     // offsets inside the prefill plan
+  size_t pre_cta = 0;     // int32 [kMaxPrefillCtas + 1]: each CTA's range of work items
   size_t pre_meta = 0;
   size_t pre_bytes = 0;
   size_t total = 0;
@@ -88,7 +89,8 @@ WsLayout ws_layout(int b, int H, int D, int rot, int64_t C) {
   L.counters = take(4 * (size_t)b * H);
   L.partials = take(4 * (size_t)(kvc::kMaxDecodeWorkers + (int64_t)b * H) * (size_t)(D + 4));
   L.pre_Pq = align_up(sizeof(kvc::PState) * (size_t)b, 16);
-  L.pre_meta = align_up(L.pre_Pq + 4 * (size_t)(b + 1), 16);
+  L.pre_cta = align_up(L.pre_Pq + 4 * (size_t)(b + 1), 16);
+  L.pre_meta = align_up(L.pre_cta + 4 * (size_t)(kvc::kMaxPrefillCtas + 1), 16);
   L.pre_bytes = L.pre_meta + 4 * (size_t)C;
   L.pre = take(L.pre_bytes);
   L.total = o;
@@ -227,6 +229,7 @@ struct kvc_cache {
   uint64_t pre_version = UINT64_MAX;
   std::vector<int32_t> pre_nq;
   int64_t pre_tiles = 0;
+  int pre_ctas = 0;
   kvc::PrefillMaps maps;
 
   kvc_cache(const kvc_config& c, int64_t C_)
@@ -884,6 +887,43 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
       qtok += n_q[s];
       Pq[s + 1] = Pq[s] + (n_q[s] + 127) / 128;
     }
+    // Work items (sequence, head, query tile) in the kernel's order -- sequence, head, the tile with
+    // the most keys first -- split into contiguous ranges of equal work (key tiles + 1 per item),
+    // one per CTA of the persistent grid: balanced, and each CTA stays on a few (sequence, head)
+    // streams whose K/V rows it re-reads from L2.
+    const int64_t n_items = (int64_t)H * Pq[b];
+    const int G = (int)std::min<int64_t>(
+        std::min(c->num_sms * kvc::prefill_ctas_per_sm(c->cfg.d_head), kvc::kMaxPrefillCtas), n_items);
+    int32_t* cta = reinterpret_cast<int32_t*>(img + c->ws.pre_cta);
+    std::vector<int32_t> work_sq;  // per (s, query tile), heads alike
+    std::vector<int> sq_seq;
+    double W = 0.0;
+    for (int s = 0; s < b; ++s) {
+      const int nqt = Pq[s + 1] - Pq[s];
+      for (int qt = nqt - 1; qt >= 0; --qt) {
+        const int64_t q_end = std::min<int64_t>(ps[s].q0 + 128 * (int64_t)(qt + 1), ps[s].len);
+        work_sq.push_back((int32_t)((q_end + 127) / 128 + 1));
+        W += (double)H * work_sq.back();
+      }
+    }
+    cta[0] = 0;
+    {
+      int c_next = 1;
+      double acc = 0.0;
+      int64_t item = 0;
+      size_t base = 0;
+      for (int s = 0; s < b; ++s) {
+        const int nqt = Pq[s + 1] - Pq[s];
+        for (int h = 0; h < H; ++h)
+          for (int k = 0; k < nqt; ++k, ++item) {
+            acc += work_sq[base + k];
+            while (c_next < G && acc >= W * c_next / G) cta[c_next++] = (int32_t)(item + 1);
+          }
+        base += nqt;
+      }
+      while (c_next <= G) cta[c_next++] = (int32_t)n_items;
+    }
+    c->pre_ctas = G;
     e = c->ring.commit(c->wsp(c->ws.pre), bytes, stream);
     if (e != cudaSuccess) return cuda_fail(e, "upload prefill plan");
     c->pre_version = c->version;
@@ -901,6 +941,7 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
   a.Pq = reinterpret_cast<const int32_t*>(c->wsp(c->ws.pre + c->ws.pre_Pq));
   a.meta = reinterpret_cast<const int32_t*>(c->wsp(c->ws.pre + c->ws.pre_meta));
   a.q = static_cast<const uint16_t*>(q);
+  a.v = static_cast<const uint16_t*>(c->cfg.v_base);
   a.out = out;
   a.c2 = (float)((double)scale * 1.4426950408889634);
   a.pos = c->cfg.pos_base;
@@ -912,7 +953,10 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
   a.status = c->bufs().status;
   a.wait_limit_ns = 2000000000ull;
   (void)D;
-  e = kvc::launch_prefill(c->geom(), c->maps, a, (int64_t)H * c->pre_tiles, stream);
+  a.n_items = (int64_t)H * c->pre_tiles;
+  a.cta_items = reinterpret_cast<const int32_t*>(c->wsp(c->ws.pre + c->ws.pre_cta));
+  a.n_ctas = c->pre_ctas;
+  e = kvc::launch_prefill(c->geom(), c->maps, a, stream);
   if (e != cudaSuccess) return cuda_fail(e, "prefill kernel");
   c->launches += 1;
   c->last_was_decode = false;

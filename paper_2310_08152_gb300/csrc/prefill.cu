@@ -21,6 +21,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -31,8 +32,11 @@
 namespace kvc {
 namespace {
 
-constexpr int kPfRows = 128;     // queries per tile (MMA M) and keys per tile (QK^T N, PV K)
-constexpr int kPfThreads = 192;  // producer warp, MMA warp, 4 softmax warps
+constexpr int kPfRows = 128;  // queries per tile (MMA M) and keys per tile (QK^T N, PV K)
+// Threads: a producer warp, an MMA warp, and NS softmax warpgroups that split each S row's 128
+// columns (NS threads per query row, one in each warpgroup).
+__host__ __device__ constexpr int pf_threads(int NS) { return 64 + 128 * NS; }
+constexpr int kPfSplit = 1;
 
 // Shared-memory geometry for head dimension D.  Q, K and V tiles are [128 rows][D] split into
 // column subtiles of SW bytes per row, the widest swizzle (128 / 64 / 32 bytes) that divides a row;
@@ -44,13 +48,24 @@ struct PfCfg {
   static constexpr int NSUB = D / SUB;
   static constexpr uint32_t SUBB = kPfRows * SW;  // bytes of one subtile
   static constexpr uint32_t TILE = kPfRows * D * 2;
-  static constexpr int NST = D <= 96 ? 3 : 2;  // K/V stages
+  // d_head 64 runs two CTAs per SM (their softmax steps interleave), each with a single S tile in
+  // TMEM and two K/V stages; larger heads run one CTA per SM with a double-buffered S tile.
+  static constexpr int CPS = D == 64 ? 2 : 1;      // CTAs per SM
+  static constexpr int SBUF = CPS == 2 ? 1 : 2;    // S tiles in TMEM
+  static constexpr int NST = CPS == 2 ? 2 : D <= 96 ? 3 : 2;  // K/V stages
   static constexpr uint32_t Q_OFF = 0;
   static constexpr uint32_t KV_OFF = TILE;
-  static constexpr uint32_t P_OFF = KV_OFF + NST * 2 * TILE;
-  static constexpr uint32_t P_BYTES = kPfRows * kPfRows * 2;
-  static constexpr uint32_t SMEM = P_OFF + P_BYTES + 1024;  // + slack to align the base to 1024
-  static constexpr uint32_t TMEM_COLS = 512;                 // S0 [0,128), S1 [128,256), O [256,256+D)
+  // Mask columns: one 16-column subtile (32-byte swizzle) appended to Q (a constant) and to every K
+  // stage (0 or a large negative number per key), so keys hidden from a whole query tile are masked
+  // by the Q.K^T product itself.
+  static constexpr uint32_t XQ_OFF = KV_OFF + NST * 2 * TILE;
+  static constexpr uint32_t XK_OFF = XQ_OFF + kPfRows * 32;
+  static constexpr uint32_t SMEM = XK_OFF + NST * kPfRows * 32 + 1024;  // + slack to align the base to 1024
+  // TMEM: SBUF S tiles of 128 columns (P, 16-bit, written over the first 64 columns of its S
+  // tile), then O0 and O1 of D columns each (alternating per item)
+  static constexpr uint32_t O_COL = SBUF * kPfRows;
+  static constexpr uint32_t TMEM_COLS = O_COL + 2 * D <= 256 ? 256 : 512;
+  static_assert(O_COL + 2 * D <= TMEM_COLS && TMEM_COLS * CPS <= 512, "TMEM budget");
   static_assert(D % 16 == 0 && SW * NSUB == 2 * D, "bad tile geometry");
   static_assert(SMEM <= 227 * 1024, "shared memory budget");
 };
@@ -86,6 +101,15 @@ __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// D (TMEM) += A (TMEM, M rows in lanes, two 16-bit elements per column) x B (shared memory).
+__device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   uint32_t* r = reinterpret_cast<uint32_t*>(v);
   asm volatile(
@@ -107,6 +131,14 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
 }
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float* v) {
   const uint32_t* r = reinterpret_cast<const uint32_t*>(v);
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st16u(uint32_t taddr, const uint32_t* r) {
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
           taddr),
@@ -158,28 +190,22 @@ struct Pack16<BF16T> {
   }
 };
 
-// RoPE (rotate-half) of a query row held in registers: pairs (e, e + HALF) for e < HALF, with the
-// rotary half-width a compile-time constant so the row stays in registers.
-template <int HALF>
-__device__ __forceinline__ void rope_rotate(float* x, int32_t pos, const float2* g) {
-#pragma unroll
-  for (int e = 0; e < HALF; ++e) {
-    float sn, cs;
-    rope_sincos(pos, g[e], &sn, &cs);
-    const float x1 = x[e], x2 = x[e + HALF];
-    x[e] = x1 * cs - x2 * sn;
-    x[e + HALF] = x2 * cs + x1 * sn;
-  }
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
 }
-// rotary_dim / 2 is a multiple of 8 in [8, D/2]
-template <int D, int HALF = D / 2>
-__device__ __forceinline__ void rope_dispatch(float* x, int half, int32_t pos, const float2* g) {
-  if constexpr (HALF >= 8) {
-    if (half == HALF)
-      rope_rotate<HALF>(x, pos, g);
-    else
-      rope_dispatch<D, HALF - 8>(x, half, pos, g);
-  }
+
+// Named barrier over the softmax warpgroups that also ANDs a flag across them.
+__device__ __forceinline__ bool bar_and(int id, int n, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 q, %1, 0;\n\tbar.red.and.pred p, %2, %3, q;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)v), "r"(id), "r"(n)
+      : "memory");
+  return r != 0;
 }
 
 // Bounded wait that also gives up as soon as another role of the CTA has given up.
@@ -200,47 +226,63 @@ __device__ __forceinline__ bool pf_wait(uint64_t* bar, uint32_t parity, const Pr
   }
 }
 
-template <typename T, int D>
-__global__ void __launch_bounds__(kPfThreads, 1)
+// One work item: query tile qt of (sequence s, head h).  Items of sequence s are
+// [H * Pq[s], H * Pq[s+1]), head-major, the tile with the most keys first.
+struct PfItem {
+  PState ps;
+  int s, h, qr0, qr_end, nk;
+  int64_t row_base;  // K/V plane row of stored row 0 of (layer, s, h)
+};
+
+__device__ __forceinline__ PfItem pf_item(const PrefillArgs& a, int64_t it) {
+  int lo = 0, hi = a.b - 1;  // last s with H * Pq[s] <= it
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if ((int64_t)a.H * a.Pq[mid] <= it)
+      lo = mid;
+    else
+      hi = mid - 1;
+  }
+  PfItem w;
+  const int nqt = a.Pq[lo + 1] - a.Pq[lo];
+  const int64_t local = it - (int64_t)a.H * a.Pq[lo];
+  w.ps = a.ps[lo];
+  w.s = lo;
+  w.h = (int)(local / nqt);
+  const int qt = nqt - 1 - (int)(local % nqt);
+  w.qr0 = w.ps.q0 + kPfRows * qt;                   // first query row of the tile
+  w.qr_end = min(w.qr0 + kPfRows, w.ps.len);        // one past its last
+  w.nk = (w.qr_end + kPfRows - 1) / kPfRows;        // key tiles [0, nk)
+  w.row_base = (int64_t)a.layer * a.H * a.C + a.seq_row0[lo] + (int64_t)w.h * a.cap[lo];
+  return w;
+}
+
+// Persistent: each CTA walks its contiguous range of items (balanced by the host); every barrier
+// phase counts tiles over all of the CTA's items, so the producer streams the next item's K/V while
+// the current one finishes, and the O accumulator alternates between two TMEM buffers per item.
+template <typename T, int D, int NS>
+__global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
     prefill_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                    const PrefillArgs a) {
   using Cf = PfCfg<D>;
-  constexpr int SW = Cf::SW, SUB = Cf::SUB, NST = Cf::NST;
+  constexpr int SW = Cf::SW, SUB = Cf::SUB, NST = Cf::NST, SBUF = Cf::SBUF;
   extern __shared__ uint8_t pf_smem_raw[];
-  __shared__ uint64_t full_bar[NST], empty_bar[NST], s_full[2], s_free[2];
+  __shared__ uint64_t full_bar[NST], empty_bar[NST], s_full[SBUF];
   __shared__ uint64_t q_full, p_full, pv_done, drain;
-  // Per stage, the tile's keys against this CTA's query tile [qr0, qr_end): khid has bit c set when
+  // Per stage, the tile's keys against its item's query tile [qr0, qr_end): khid has bit c set when
   // key c's bound holds for every query of the tile (hid >= qr_end - 1); klist holds the keys whose
   // bound falls inside it (qr0 <= hid < qr_end - 1: a span closing among the queries), kn of them.
   __shared__ uint4 khid[NST];
   __shared__ int2 klist[NST][kPfRows];
   __shared__ int32_t kn[NST];
+  __shared__ int32_t kslow[NST];  // the tile needs the per-key rule (else its mask column decides)
+  __shared__ float xbuf[2 * NS * kPfRows];
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
 
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(pf_smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  // work item: blocks of sequence s are [H * Pq[s], H * Pq[s+1]), head-major, longest tile first
-  const int64_t bid = blockIdx.x;
-  int lo = 0, hi = a.b - 1;  // last s with H * Pq[s] <= bid
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if ((int64_t)a.H * a.Pq[mid] <= bid)
-      lo = mid;
-    else
-      hi = mid - 1;
-  }
-  const int s = lo;
-  const int nqt = a.Pq[s + 1] - a.Pq[s];
-  const int64_t local = bid - (int64_t)a.H * a.Pq[s];
-  const int h = (int)(local / nqt);
-  const int qt = nqt - 1 - (int)(local % nqt);
-  const PState ps = a.ps[s];
-  const int qr0 = ps.q0 + kPfRows * qt;                 // first query row of the tile
-  const int qr_end = min(qr0 + kPfRows, ps.len);        // one past its last
-  const int nk = (qr_end + kPfRows - 1) / kPfRows;      // key tiles [0, nk)
-  const int64_t row_base = (int64_t)a.layer * a.H * a.C + a.seq_row0[s] + (int64_t)h * a.cap[s];
+  const int64_t it0 = a.cta_items[blockIdx.x], it1 = a.cta_items[blockIdx.x + 1];  // this CTA's items
 
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_slot)),
@@ -253,12 +295,9 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       mbar_init(&full_bar[i], 32);
       mbar_init(&empty_bar[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&s_full[i], 1);
-      mbar_init(&s_free[i], 128);
-    }
-    mbar_init(&q_full, 128);
-    mbar_init(&p_full, 128);
+    for (int i = 0; i < SBUF; ++i) mbar_init(&s_full[i], 1);
+    mbar_init(&q_full, 128 * NS);
+    mbar_init(&p_full, 128 * NS);
     mbar_init(&pv_done, 1);
     mbar_init(&drain, 1);
     abort_flag = 0;
@@ -271,65 +310,91 @@ __global__ void __launch_bounds__(kPfThreads, 1)
 
   if (warp == 0) {
     // ---------------- producer ----------------
-    int issued = 0;
+    int64_t g = 0;  // tiles issued
     bool ok = true;
-    for (int j = 0; j < nk; ++j) {
-      const int st = j % NST;
-      if (j >= NST && !pf_wait(&empty_bar[st], ((j / NST) - 1) & 1, a, &abort_flag)) {
-        ok = false;
-        break;
-      }
-      if (lane == 0) {
-        mbar_expect_tx(&full_bar[st], 2 * Cf::TILE);
-        const int y = (int)(row_base + (int64_t)kPfRows * j);
-        const uint32_t kt = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE);
-#pragma unroll
-        for (int u = 0; u < Cf::NSUB; ++u) {
-          tma_load_2d(kt + u * Cf::SUBB, &tm_k, u * SUB, y, &full_bar[st]);
-          tma_load_2d(kt + Cf::TILE + u * Cf::SUBB, &tm_v, u * SUB, y, &full_bar[st]);
+    for (int64_t it = it0; ok && it < it1; ++it) {
+      const PfItem w = pf_item(a, it);
+      for (int j = 0; j < w.nk; ++j, ++g) {
+        const int st = (int)(g % NST);
+        if (g >= NST && !pf_wait(&empty_bar[st], (uint32_t)((g / NST) - 1) & 1, a, &abort_flag)) {
+          ok = false;
+          break;
         }
-      }
-      ++issued;
-      // per-key mask bounds of the tile ((hid << 1) | is_cl; rows past the stored ones: invisible)
-      // sorted into the classes above; the causal part (i <= iq) is left to each query
-      uint32_t ok_w[4];
-      int n_part = 0;
+        if (lane == 0) {
+          mbar_expect_tx(&full_bar[st], 2 * Cf::TILE);
+          const int y = (int)(w.row_base + (int64_t)kPfRows * j);
+          const uint32_t kt = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE);
 #pragma unroll
-      for (int w4 = 0; w4 < 4; ++w4) {
-        const int c = lane + 32 * w4;
-        const int i = kPfRows * j + c;
-        const int hid = (i < ps.len ? a.meta[ps.moff + i] : -2) >> 1;
-        ok_w[w4] = __ballot_sync(0xFFFFFFFFu, hid >= qr_end - 1);
-        const bool part = hid >= qr0 && hid < qr_end - 1;
-        const uint32_t pb = __ballot_sync(0xFFFFFFFFu, part);
-        if (part) klist[st][n_part + __popc(pb & ((1u << lane) - 1u))] = make_int2(c, hid);
-        n_part += __popc(pb);
+          for (int u = 0; u < Cf::NSUB; ++u) {
+            tma_load_2d(kt + u * Cf::SUBB, &tm_k, u * SUB, y, &full_bar[st]);
+            tma_load_2d(kt + Cf::TILE + u * Cf::SUBB, &tm_v, u * SUB, y, &full_bar[st]);
+          }
+        }
+        // per-key mask bounds of the tile ((hid << 1) | is_cl; rows past the stored ones: invisible)
+        // sorted into the classes above; the causal part (i <= iq) is left to each query
+        uint32_t ok_w[4];
+        bool none[4];
+        int n_part = 0;
+#pragma unroll
+        for (int w4 = 0; w4 < 4; ++w4) {
+          const int c = lane + 32 * w4;
+          const int i = kPfRows * j + c;
+          const int hid = (i < w.ps.len ? a.meta[w.ps.moff + i] : -2) >> 1;
+          none[w4] = i >= w.qr_end || hid < w.qr0;  // visible to no query of the tile
+          ok_w[w4] = __ballot_sync(0xFFFFFFFFu, hid >= w.qr_end - 1);
+          const bool part = hid >= w.qr0 && hid < w.qr_end - 1;
+          const uint32_t pb = __ballot_sync(0xFFFFFFFFu, part);
+          if (part) klist[st][n_part + __popc(pb & ((1u << lane) - 1u))] = make_int2(c, hid);
+          n_part += __popc(pb);
+        }
+        if (lane == 0) {
+          khid[st] = make_uint4(ok_w[0], ok_w[1], ok_w[2], ok_w[3]);
+          // per-key masking is needed when a key's visibility differs between the tile's queries,
+          // or when the tile holds rows past the stored ones (their K may be anything)
+          kn[st] = n_part;
+          kslow[st] = n_part > 0 || kPfRows * (j + 1) > w.ps.len || kPfRows * (j + 1) > w.qr0 + 1;
+        }
+        // mask column of the tile: a large negative number for keys no query of the tile may see
+#pragma unroll
+        for (int w4 = 0; w4 < 4; ++w4) {
+          const int c = lane + 32 * w4;
+          const uint32_t x0 = none[w4] ? (uint32_t)T::r(-32768.f) : 0u;
+          const uint32_t row = smem_addr(sm + Cf::XK_OFF + st * kPfRows * 32) + c * 32;
+          const uint32_t sw = (c >> 2) & 1;  // 32-byte swizzle: the two 16-byte halves swap every 4 rows
+          st_shared_v4(row + 16 * sw, x0, 0u, 0u, 0u);
+          st_shared_v4(row + 16 * (sw ^ 1), 0u, 0u, 0u, 0u);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        mbar_arrive(&full_bar[st]);
       }
-      if (lane == 0) {
-        khid[st] = make_uint4(ok_w[0], ok_w[1], ok_w[2], ok_w[3]);
-        kn[st] = n_part;
-      }
-      __syncwarp();
-      mbar_arrive(&full_bar[st]);
     }
     if (!ok && lane == 0) {
       // let the copies already issued land before the CTA exits
-      for (int j = max(0, issued - NST); j < issued; ++j) mbar_wait_bounded(&full_bar[j % NST], (j / NST) & 1, 100000000ull);
+      for (int64_t t = g > NST ? g - NST : 0; t < g; ++t)
+        mbar_wait_bounded(&full_bar[t % NST], (uint32_t)(t / NST) & 1, 100000000ull);
     }
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       constexpr uint32_t idS = mma_idesc(Pack16<T>::kType, 0, kPfRows, kPfRows);
       constexpr uint32_t idO = mma_idesc(Pack16<T>::kType, 1, kPfRows, D);
-      const uint32_t q_s = smem_addr(sm + Cf::Q_OFF), p_s = smem_addr(sm + Cf::P_OFF);
-      bool ok = pf_wait(&q_full, 0, a, &abort_flag);
-      tc_fence_after();
-      for (int j = 0; ok && j <= nk; ++j) {
-        if (j < nk) {
-          const int st = j % NST, sb = j & 1;
-          ok = pf_wait(&full_bar[st], (j / NST) & 1, a, &abort_flag);
-          if (ok && j >= 2) ok = pf_wait(&s_free[sb], ((j - 2) >> 1) & 1, a, &abort_flag);
-          if (!ok) break;
+      const uint32_t q_s = smem_addr(sm + Cf::Q_OFF);
+      const uint32_t xq_s = smem_addr(sm + Cf::XQ_OFF), xk_s = smem_addr(sm + Cf::XK_OFF);
+      int64_t g = 0;
+      uint32_t k = 0;
+      bool ok = true;
+      for (int64_t it = it0; ok && it < it1; ++it, ++k) {
+        const int nk = pf_item(a, it).nk;
+        ok = pf_wait(&q_full, k & 1, a, &abort_flag);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t o_t = tmem + Cf::O_COL + (k & 1) * D;
+        // S = Q K^T of tile gj into its S tile, which last held P of tile gj - SBUF: the P.V reading
+        // it was issued before (tcgen05.mma from one thread run in issue order)
+        auto issue_qk = [&](int64_t gj) -> bool {
+          const int st = (int)(gj % NST), sb = (int)(gj % SBUF);
+          if (!pf_wait(&full_bar[st], (uint32_t)(gj / NST) & 1, a, &abort_flag)) return false;
           tc_fence_after();
           const uint32_t k_s = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE);
 #pragma unroll
@@ -338,215 +403,335 @@ __global__ void __launch_bounds__(kPfThreads, 1)
             tc_mma(tmem + sb * kPfRows, smem_desc(q_s + off, 16, 8 * SW, SW), smem_desc(k_s + off, 16, 8 * SW, SW),
                    idS, kk > 0);
           }
+          // + the mask column: 256 x (0 or -32768) per key
+          tc_mma(tmem + sb * kPfRows, smem_desc(xq_s, 16, 8 * 32, 32),
+                 smem_desc(xk_s + st * kPfRows * 32, 16, 8 * 32, 32), idS, 1);
           tc_commit(&s_full[sb]);
-        }
-        if (j >= 1) {
-          const int jj = j - 1, st = jj % NST;
-          ok = pf_wait(&p_full, jj & 1, a, &abort_flag);
-          if (!ok) break;
+          return true;
+        };
+        // O += P V of tile gp (P in its S tile, 8 TMEM columns per 16 keys); first of the item: O = P V
+        auto issue_pv = [&](int64_t gp, bool first) -> bool {
+          const int st = (int)(gp % NST);
+          if (!pf_wait(&p_full, (uint32_t)gp & 1, a, &abort_flag)) return false;
           tc_fence_after();
           const uint32_t v_s = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE + Cf::TILE);
+          const uint32_t p_t = tmem + (uint32_t)(gp % SBUF) * kPfRows;
 #pragma unroll
-          for (int kk = 0; kk < kPfRows / 16; ++kk) {
-            tc_mma(tmem + 2 * kPfRows, smem_desc(p_s + (kk >> 2) * (kPfRows * 128) + (kk & 3) * 32, 16, 1024, 128),
-                   smem_desc(v_s + kk * 16 * SW, Cf::SUBB, 8 * SW, SW), idO, (jj > 0 || kk > 0));
-          }
+          for (int kk = 0; kk < kPfRows / 16; ++kk)
+            tc_mma_ts(o_t, p_t + 8 * kk, smem_desc(v_s + kk * 16 * SW, Cf::SUBB, 8 * SW, SW), idO, (!first || kk > 0));
           tc_commit(&pv_done);
           tc_commit(&empty_bar[st]);
+          return true;
+        };
+        for (int j = 0; ok && j <= nk; ++j) {
+          if (SBUF == 2) {  // Q K^T of the next tile runs while the softmax of this one does
+            if (j < nk) ok = issue_qk(g + j);
+            if (ok && j >= 1) ok = issue_pv(g + j - 1, j == 1);
+          } else {          // one S tile: P.V of the previous tile first
+            if (j >= 1) ok = issue_pv(g + j - 1, j == 1);
+            if (ok && j < nk) ok = issue_qk(g + j);
+          }
         }
+        g += nk;
       }
       // every MMA issued above has completed once this phase does
       tc_commit(&drain);
       mbar_wait_bounded(&drain, 0, a.wait_limit_ns);
     }
   } else {
-    // ---------------- softmax: one query row per thread ----------------
+    // ---------------- softmax: NS threads per query row ----------------
+    constexpr int CW = kPfRows / NS;  // S columns of one thread
+    constexpr int NSM = 128 * NS;     // softmax threads (named barrier 1)
     const int quarter = warp & 3;
+    const int hs = (warp - 2) >> 2;     // which column slice of the row
     const int r = quarter * 32 + lane;  // tile row == TMEM lane
     const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
-    const int iq = qr0 + r;  // stored row of this query
-    const bool valid = iq < qr_end;
-    const int64_t out_row = valid ? ((int64_t)(ps.qtok + (iq - ps.q0)) * a.H + h) * D : 0;
-    {
-      // the query row, rotated at its position (RoPE), rounded to the cache type, into the K-major tile
-      float x[D];
-      if (valid) {
-        const uint4* src = reinterpret_cast<const uint4*>(a.q + out_row);
+    const float c2 = a.c2;
+    float* xmax = xbuf;  // [2][NS][128] row-maximum exchange; [NS][128] row sums at the end
+    // the query row of item w, rotated at its position (RoPE, pairs (e, e + rot/2)), rounded to the
+    // cache type, into the K-major tile; 8 columns at a time
+    auto write_q = [&](const PfItem& w) {
+      if (hs == 0) {
+        const int iq = w.qr0 + r;
+        const bool valid = iq < w.qr_end;
+        const uint32_t q_s = smem_addr(sm + Cf::Q_OFF);
+        const int64_t row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : 0;
+        const uint4* src = reinterpret_cast<const uint4*>(a.q + row);
+        const int half = a.rot / 2;
+        const int32_t qpos = (valid && half > 0) ? a.pos[a.off[w.s] + iq] : 0;
+        auto load8 = [&](int c8, float* x) {
+          if (valid) {
+            const uint4 u = __ldg(src + c8);
+            const uint32_t wd[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float2 f = T::f2(wd[e]);
+              x[2 * e] = f.x;
+              x[2 * e + 1] = f.y;
+            }
+          } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[e] = 0.f;
+          }
+        };
+        auto store8 = [&](int c8, const float* x) {
+          const int e0 = c8 * 8;
+          const int u = e0 / SUB, cw = (e0 % SUB) / 8;
+          const int phys = cw ^ ((r * SW >> 7) & (SW / 16 - 1));
+          st_shared_v4(q_s + u * Cf::SUBB + r * SW + phys * 16, Pack16<T>::two(x[0], x[1]),
+                       Pack16<T>::two(x[2], x[3]), Pack16<T>::two(x[4], x[5]), Pack16<T>::two(x[6], x[7]));
+        };
 #pragma unroll
         for (int c8 = 0; c8 < D / 8; ++c8) {
-          const uint4 u = __ldg(src + c8);
-          const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+          const int e0 = 8 * c8;
+          if (e0 < half) {
+            float x1[8], x2[8];
+            load8(c8, x1);
+            load8(c8 + half / 8, x2);
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 f = T::f2(w[e]);
-            x[c8 * 8 + 2 * e] = f.x;
-            x[c8 * 8 + 2 * e + 1] = f.y;
+            for (int e = 0; e < 8; ++e) {
+              float sn, cs;
+              rope_sincos(qpos, a.rope_g[e0 + e], &sn, &cs);
+              const float y1 = x1[e] * cs - x2[e] * sn;
+              x2[e] = x2[e] * cs + x1[e] * sn;
+              x1[e] = y1;
+            }
+            store8(c8, x1);
+            store8(c8 + half / 8, x2);
+          } else if (e0 >= 2 * half) {
+            float x[8];
+            load8(c8, x);
+            store8(c8, x);
           }
         }
-        if (a.rot > 0) rope_dispatch<D>(x, a.rot / 2, a.pos[a.off[s] + iq], a.rope_g);
-      } else {
-#pragma unroll
-        for (int e = 0; e < D; ++e) x[e] = 0.f;
       }
-      const uint32_t q_s = smem_addr(sm + Cf::Q_OFF);
-#pragma unroll
-      for (int c8 = 0; c8 < D / 8; ++c8) {
-        const int e0 = c8 * 8;
-        const int u = e0 / SUB, cw = (e0 % SUB) / 8;
-        const int phys = cw ^ ((r * SW >> 7) & (SW / 16 - 1));
-        st_shared_v4(q_s + u * Cf::SUBB + r * SW + phys * 16, Pack16<T>::two(x[e0], x[e0 + 1]),
-                     Pack16<T>::two(x[e0 + 2], x[e0 + 3]), Pack16<T>::two(x[e0 + 4], x[e0 + 5]),
-                     Pack16<T>::two(x[e0 + 6], x[e0 + 7]));
-      }
+      fence_proxy_async_smem();
+      mbar_arrive(&q_full);
+    };
+
+    if (hs == 0) {
+      // the constant half of the mask column: 256 in column 0 of every query row
+      const uint32_t row = smem_addr(sm + Cf::XQ_OFF) + r * 32;
+      const uint32_t sw = (r >> 2) & 1;
+      st_shared_v4(row + 16 * sw, (uint32_t)T::r(256.f), 0u, 0u, 0u);
+      st_shared_v4(row + 16 * (sw ^ 1), 0u, 0u, 0u, 0u);
     }
-    fence_proxy_async_smem();
-    mbar_arrive(&q_full);
-    const bool cl_q = valid && (a.meta[ps.moff + iq] & 1);
-    const float c2 = a.c2;
-    float m = -INFINITY, l = 0.f;
     bool ok = true;
-    const uint32_t p_row = smem_addr(sm + Cf::P_OFF) + r * 128;
-    for (int j = 0; j < nk; ++j) {
-      const int sb = j & 1, st = j % NST;
-      // the S tile, and (acquired from the producer directly) the stage's mask bounds; the stage's
-      // barrier cannot move to its next phase before this thread releases P of this tile.  Warp-
-      // uniform outcome: the tcgen05 loads and stores below are .sync.aligned.
-      ok = pf_wait(&s_full[sb], (j >> 1) & 1, a, &abort_flag) &&
-           pf_wait(&full_bar[st], (j / NST) & 1, a, &abort_flag);
-      if (!__all_sync(0xFFFFFFFFu, ok)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      float sv[kPfRows];
+    int64_t g = 0;  // tiles consumed
+    uint32_t k = 0;  // items done
+    int64_t it = it0;
+    PfItem w{};
+    if (it < it1) {
+      w = pf_item(a, it);
+      write_q(w);
+    }
+    while (it < it1) {
+      const int iq = w.qr0 + r;  // stored row of this query
+      const bool valid = iq < w.qr_end;
+      const bool cl_q = valid && (a.meta[w.ps.moff + iq] & 1);
+      const uint32_t o_t = tl + Cf::O_COL + (k & 1) * D;
+      float m = -INFINITY, l = 0.f;
+      for (int j = 0; j < w.nk; ++j) {
+        const int64_t gj = g + j;
+        const int sb = (int)(gj % SBUF), st = (int)(gj % NST);
+        // the S tile, and (acquired from the producer directly) the stage's mask bounds; the stage's
+        // barrier cannot move to its next phase before this thread releases P of this tile
+        ok = ok && pf_wait(&s_full[sb], (uint32_t)(gj / SBUF) & 1, a, &abort_flag) &&
+             pf_wait(&full_bar[st], (uint32_t)(gj / NST) & 1, a, &abort_flag);
+        const bool wok = __all_sync(0xFFFFFFFFu, ok);  // tcgen05.ld / st are warp-collective
+        float sv[CW];
+        if (wok) {
+          tc_fence_after();
 #pragma unroll
-      for (int c = 0; c < kPfRows; c += 32) tmem_ld32(tl + sb * kPfRows + c, sv + c);
-      tmem_wait_ld();
-      tc_fence_before();
-      mbar_arrive(&s_free[sb]);
-      const int kb = kPfRows * j;
-      // visibility of the tile's keys to this query as four 32-bit words: the causal prefix
-      // (key row <= iq) and the tile-wide bound words, plus the listed keys whose bound admits iq; a
-      // <CL> query sees only its own row
-      const int t = iq - kb;  // last visible column
-      uint32_t v0, v1, v2, v3;
-      {
-        auto prefix = [t](int w) -> uint32_t {
-          const int n = t - 32 * w + 1;  // columns of word w at or before t
-          return n <= 0 ? 0u : n >= 32 ? 0xFFFFFFFFu : (1u << n) - 1u;
-        };
-        if (cl_q) {
-          auto one = [t](int w) -> uint32_t { return (t >> 5) == w ? 1u << (t & 31) : 0u; };
-          v0 = one(0), v1 = one(1), v2 = one(2), v3 = one(3);
+          for (int c = 0; c < CW; c += 32) tmem_ld32(tl + sb * kPfRows + hs * CW + c, sv + c);
+          tmem_wait_ld();
+          tc_fence_before();
         } else {
+#pragma unroll
+          for (int c = 0; c < CW; ++c) sv[c] = 0.f;
+        }
+        const int kb = kPfRows * j;
+        if (kslow[st]) {
+          // visibility of the tile's keys to this query as four 32-bit words: the causal prefix (key
+          // row <= iq) with the tile-wide bound words plus the listed keys whose bound admits iq.
+          // (<CL> queries take their own value row in the epilogue.)  Other tiles are masked by
+          // their mask column alone.
+          const int t = iq - kb;  // last visible column
+          auto prefix = [t](int wd) -> uint32_t {
+            const int n = t - 32 * wd + 1;  // columns of word wd at or before t
+            return n <= 0 ? 0u : n >= 32 ? 0xFFFFFFFFu : (1u << n) - 1u;
+          };
           const uint4 hw = khid[st];
-          v0 = hw.x, v1 = hw.y, v2 = hw.z, v3 = hw.w;
+          uint32_t v0 = hw.x, v1 = hw.y, v2 = hw.z, v3 = hw.w;
           const int np = kn[st];
           for (int e = 0; e < np; ++e) {
             const int2 ent = klist[st][e];
             if (ent.y >= iq) {
               const uint32_t bit = 1u << (ent.x & 31);
-              const int w = ent.x >> 5;
-              v0 |= w == 0 ? bit : 0u;
-              v1 |= w == 1 ? bit : 0u;
-              v2 |= w == 2 ? bit : 0u;
-              v3 |= w == 3 ? bit : 0u;
+              const int wd = ent.x >> 5;
+              v0 |= wd == 0 ? bit : 0u;
+              v1 |= wd == 1 ? bit : 0u;
+              v2 |= wd == 2 ? bit : 0u;
+              v3 |= wd == 3 ? bit : 0u;
             }
           }
           v0 &= prefix(0), v1 &= prefix(1), v2 &= prefix(2), v3 &= prefix(3);
+          // this thread's words: columns [hs * CW, hs * CW + CW)
+          uint32_t vw[CW / 32];
+#pragma unroll
+          for (int q = 0; q < CW / 32; ++q) {
+            const int wd = hs * (CW / 32) + q;
+            vw[q] = wd == 0 ? v0 : wd == 1 ? v1 : wd == 2 ? v2 : v3;
+          }
+#pragma unroll
+          for (int c = 0; c < CW; ++c) sv[c] = (vw[c >> 5] >> (c & 31)) & 1u ? sv[c] : -INFINITY;
         }
-      }
-      if ((v0 & v1 & v2 & v3) != 0xFFFFFFFFu) {
+        // row max: a tree over this slice, then across the NS slices of the row
+        float mx8[8];
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          sv[e] = (v0 >> e) & 1u ? sv[e] : -INFINITY;
-          sv[32 + e] = (v1 >> e) & 1u ? sv[32 + e] : -INFINITY;
-          sv[64 + e] = (v2 >> e) & 1u ? sv[64 + e] : -INFINITY;
-          sv[96 + e] = (v3 >> e) & 1u ? sv[96 + e] : -INFINITY;
+        for (int u = 0; u < 8; ++u) mx8[u] = sv[u];
+#pragma unroll
+        for (int c = 8; c + 16 <= CW; c += 16)
+#pragma unroll
+          for (int u = 0; u < 8; ++u) mx8[u] = max3(mx8[u], sv[c + u], sv[c + 8 + u]);
+        if (CW % 16 == 8) {
+#pragma unroll
+          for (int u = 0; u < 8; ++u) mx8[u] = fmaxf(mx8[u], sv[CW - 8 + u]);
         }
-      }
-      // row max: a tree over 8 partial maxima keeps the dependency chains short
-      float mx8[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) mx8[u] = sv[u];
-#pragma unroll
-      for (int c = 8; c < kPfRows; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], sv[c]);
-      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-      // Reference maximum: moved only when the row maximum grows by more than 2^8 (log2 units), so O
-      // is rescaled rarely; P stays below 2^8 and its scale cancels exactly in O / l.
-      const float cand = mx * c2;
-      const bool move = cand > m + 8.f;
-      const float m_new = move ? cand : m;
-      const float ref = m_new == -INFINITY ? 0.f : m_new;
-      uint32_t pk[kPfRows / 2];
-      float rs8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int c = 0; c < kPfRows; c += 2) {
-        const float p0 = ex2(fmaf(sv[c], c2, -ref));
-        const float p1 = ex2(fmaf(sv[c + 1], c2, -ref));
-        rs8[(c >> 1) & 7] += p0 + p1;
-        pk[c / 2] = Pack16<T>::two(p0, p1);
-      }
-      const float rs = ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
-      const float alpha = !move ? 1.f : (m == -INFINITY ? 0.f : ex2(m - ref));
-      l = l * alpha + rs;
-      if (j >= 1) {
-        // PV of the previous tile is complete: O may be rescaled and the P tile rewritten
-        ok = pf_wait(&pv_done, (j - 1) & 1, a, &abort_flag);
-        if (!__all_sync(0xFFFFFFFFu, ok)) {
+        float mx = max3(max3(mx8[0], mx8[1], mx8[2]), max3(mx8[3], mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]));
+        if (NS > 1) xmax[((gj & 1) * NS + hs) * kPfRows + r] = mx;
+        // every softmax thread passes this barrier: the exit decision is taken by all of them at once
+        if (!bar_and(1, NSM, ok)) {
           ok = false;
           break;
         }
-        tc_fence_after();
-        if (__any_sync(0xFFFFFFFFu, alpha != 1.f)) {
+        if (NS > 1) {
 #pragma unroll
-          for (int u = 0; u < D / 16; ++u) {
-            float o[16];
-            tmem_ld16(tl + 2 * kPfRows + 16 * u, o);
-            tmem_wait_ld();
-#pragma unroll
-            for (int e = 0; e < 16; ++e) o[e] *= alpha;
-            tmem_st16(tl + 2 * kPfRows + 16 * u, o);
-          }
-          tmem_wait_st();
+          for (int q = 0; q < NS; ++q) mx = fmaxf(mx, xmax[((gj & 1) * NS + q) * kPfRows + r]);
         }
-      }
+        // Reference maximum: moved only when the row maximum grows by more than 2^8 (log2 units), so
+        // O is rescaled rarely; P stays below 2^8 and its scale cancels exactly in O / l.
+        const float cand = mx * c2;
+        const bool move = cand > m + 8.f;
+        const float m_new = move ? cand : m;
+        const float ref = m_new == -INFINITY ? 0.f : m_new;
+        uint32_t pk[CW / 2];
+        float2 rs4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+        const float2 c2v = make_float2(c2, c2), nref = make_float2(-ref, -ref);
 #pragma unroll
-      for (int c8 = 0; c8 < kPfRows / 8; ++c8) {
-        const int phys = (c8 & 7) ^ (r & 7);
-        st_shared_v4(p_row + (c8 >> 3) * (kPfRows * 128) + phys * 16, pk[4 * c8], pk[4 * c8 + 1], pk[4 * c8 + 2],
-                     pk[4 * c8 + 3]);
-      }
-      if (kb + kPfRows > ps.len && kb + r >= ps.len) {
-        // a V row past the stored rows (stale or another stream's): zero it so 0 * V stays 0
-        const uint32_t v_row = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE + Cf::TILE) + r * SW;
+        for (int c = 0; c < CW; c += 2) {
+          const float2 x = __ffma2_rn(make_float2(sv[c], sv[c + 1]), c2v, nref);
+          const float2 p = make_float2(ex2(x.x), ex2(x.y));
+          rs4[(c >> 1) & 3] = __fadd2_rn(rs4[(c >> 1) & 3], p);
+          pk[c / 2] = Pack16<T>::two(p.x, p.y);
+        }
+        const float rs = ((rs4[0].x + rs4[0].y) + (rs4[1].x + rs4[1].y)) + ((rs4[2].x + rs4[2].y) + (rs4[3].x + rs4[3].y));
+        const float alpha = !move ? 1.f : (m == -INFINITY ? 0.f : ex2(m - ref));
+        l = l * alpha + rs;  // this slice's part of the row sum
+        // pv_done phases are consumed one by one, each while it is the only one that can be pending
+        // (the next P.V waits for this tile's P): phase gj - 1 during tile j >= 1, before P is
+        // released, early when O has to be rescaled; an item's last phase in its epilogue.
+        bool pv_waited = false;
+        if (j >= 1 && __any_sync(0xFFFFFFFFu, alpha != 1.f)) {
+          ok = pf_wait(&pv_done, (uint32_t)(gj - 1) & 1, a, &abort_flag);
+          pv_waited = true;
+          if (__all_sync(0xFFFFFFFFu, ok)) {
+            tc_fence_after();
 #pragma unroll
-        for (int u = 0; u < Cf::NSUB; ++u)
+            for (int u = 0; u < D / 16; ++u) {
+              if (u % NS != hs) continue;
+              float o[16];
+              tmem_ld16(o_t + 16 * u, o);
+              tmem_wait_ld();
 #pragma unroll
-          for (int b16 = 0; b16 < SW / 16; ++b16) st_shared_v4(v_row + u * Cf::SUBB + b16 * 16, 0, 0, 0, 0);
+              for (int e = 0; e < 16; ++e) o[e] *= alpha;
+              tmem_st16(o_t + 16 * u, o);
+            }
+          }
+        }
+        // P (16-bit pairs) over the first half of this tile's S columns, row r in lane r
+        if (__all_sync(0xFFFFFFFFu, ok)) {
+#pragma unroll
+          for (int q = 0; q < CW / 32; ++q) tmem_st16u(tl + sb * kPfRows + hs * (CW / 2) + 16 * q, pk + 16 * q);
+        }
+        tmem_wait_st();
+        if (kb + kPfRows > w.ps.len && kb + r >= w.ps.len) {
+          // a V row past the stored rows (stale or another stream's): zero it so 0 * V stays 0
+          const uint32_t v_row = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE + Cf::TILE) + r * SW;
+#pragma unroll
+          for (int u = 0; u < Cf::NSUB; ++u) {
+            if (u % NS != hs) continue;
+#pragma unroll
+            for (int b16 = 0; b16 < SW / 16; ++b16) st_shared_v4(v_row + u * Cf::SUBB + b16 * 16, 0, 0, 0, 0);
+          }
+          fence_proxy_async_smem();
+        }
+        if (j >= 1 && !pv_waited) ok = pf_wait(&pv_done, (uint32_t)(gj - 1) & 1, a, &abort_flag) && ok;
+        tc_fence_before();
+        mbar_arrive(&p_full);
+        m = m_new;
       }
-      fence_proxy_async_smem();
-      tc_fence_before();
-      mbar_arrive(&p_full);
-      m = m_new;
-    }
-    if (ok) ok = pf_wait(&pv_done, (nk - 1) & 1, a, &abort_flag);
-    if (__all_sync(0xFFFFFFFFu, ok)) {
+      // a wait that ran out after the tile loop's last barrier: decided by every thread together
+      if (!bar_and(1, NSM, ok)) {
+        ok = false;
+        break;
+      }
+      g += w.nk;
+      // the next item's queries go in as soon as this item's last S tile is read (every Q K^T of
+      // this item is complete), so its first tiles overlap this item's epilogue
+      const int64_t next = it + 1;
+      PfItem wn{};
+      if (next < it1) {
+        wn = pf_item(a, next);
+        write_q(wn);
+      }
+      // epilogue: O / l, with l summed over the NS slices of the row
+      ok = pf_wait(&pv_done, (uint32_t)(g - 1) & 1, a, &abort_flag);
+      if (NS > 1) xmax[hs * kPfRows + r] = l;
+      if (!bar_and(1, NSM, ok)) {
+        ok = false;
+        break;
+      }
+      float lt = l;
+      if (NS > 1) {
+        lt = 0.f;
+#pragma unroll
+        for (int q = 0; q < NS; ++q) lt += xmax[q * kPfRows + r];
+      }
       tc_fence_after();
-      const float inv = 1.f / l;
+      const float inv = 1.f / lt;
+      const int64_t out_row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : 0;
 #pragma unroll
       for (int u = 0; u < D / 16; ++u) {
+        if (u % NS != hs) continue;
         float o[16];
-        tmem_ld16(tl + 2 * kPfRows + 16 * u, o);
+        tmem_ld16(o_t + 16 * u, o);
         tmem_wait_ld();
         if (valid) {
           float4* dst = reinterpret_cast<float4*>(a.out + out_row + 16 * u);
+          if (cl_q) {
+            // Sec. 3.1: a <CL> attends only to itself, so its output is its own value row
+            const uint4* vsrc = reinterpret_cast<const uint4*>(a.v + (w.row_base + iq) * D + 16 * u);
 #pragma unroll
-          for (int e = 0; e < 4; ++e)
-            dst[e] = make_float4(o[4 * e] * inv, o[4 * e + 1] * inv, o[4 * e + 2] * inv, o[4 * e + 3] * inv);
+            for (int e2 = 0; e2 < 2; ++e2) {
+              const uint4 vv = __ldg(vsrc + e2);
+              const float2 f0 = T::f2(vv.x), f1 = T::f2(vv.y), f2 = T::f2(vv.z), f3 = T::f2(vv.w);
+              dst[2 * e2] = make_float4(f0.x, f0.y, f1.x, f1.y);
+              dst[2 * e2 + 1] = make_float4(f2.x, f2.y, f3.x, f3.y);
+            }
+          } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              dst[e] = make_float4(o[4 * e] * inv, o[4 * e + 1] * inv, o[4 * e + 2] * inv, o[4 * e + 3] * inv);
+          }
         }
       }
+      tc_fence_before();
+      // the row sums are read before the next item's first maximum exchange reuses the buffer
+      bar_and(1, NSM, true);
+      it = next;
+      w = wn;
+      ++k;
     }
   }
   tc_fence_before();
@@ -582,7 +767,7 @@ template <typename T, int D>
 cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int64_t grid, cudaStream_t stream) {
   static bool attr_set = false;  // per instantiation; setting it twice is harmless
   if (!attr_set) {
-    const cudaError_t e = cudaFuncSetAttribute(prefill_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    const cudaError_t e = cudaFuncSetAttribute(prefill_kernel<T, D, kPfSplit>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)PfCfg<D>::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
@@ -590,7 +775,7 @@ cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int6
   CUtensorMap mk, mv;
   std::memcpy(&mk, maps.k, sizeof mk);
   std::memcpy(&mv, maps.v, sizeof mv);
-  prefill_kernel<T, D><<<(unsigned)grid, kPfThreads, PfCfg<D>::SMEM, stream>>>(mk, mv, a);
+  prefill_kernel<T, D, kPfSplit><<<(unsigned)grid, pf_threads(kPfSplit), PfCfg<D>::SMEM, stream>>>(mk, mv, a);
   return cudaGetLastError();
 }
 
@@ -611,9 +796,19 @@ cudaError_t encode_prefill_maps(const Geometry& g, const Buffers& buf, PrefillMa
   return e;
 }
 
-cudaError_t launch_prefill(const Geometry& g, const PrefillMaps& maps, const PrefillArgs& a, int64_t grid,
-                           cudaStream_t stream) {
-  if (grid <= 0) return cudaSuccess;
+int prefill_ctas_per_sm(int D) {
+  switch (D) {
+    case 64: return PfCfg<64>::CPS;
+    case 80: return PfCfg<80>::CPS;
+    case 96: return PfCfg<96>::CPS;
+    case 128: return PfCfg<128>::CPS;
+    default: return 1;
+  }
+}
+
+cudaError_t launch_prefill(const Geometry& g, const PrefillMaps& maps, const PrefillArgs& a, cudaStream_t stream) {
+  if (a.n_items <= 0 || a.n_ctas <= 0) return cudaSuccess;
+  const int64_t grid = a.n_ctas;  // persistent: at most one CTA per SM
   const bool bf = g.dtype == 1;
   switch (g.D) {
     case 64:
