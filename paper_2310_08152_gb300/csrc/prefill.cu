@@ -257,6 +257,11 @@ __device__ __forceinline__ PfItem pf_item(const PrefillArgs& a, int64_t it) {
   return w;
 }
 
+// Key tile of the j-th step of item it: consecutive items run their key tiles in opposite
+// directions, so an item starts on the tiles its predecessor (same (sequence, head), most often)
+// read last, while they are still in L2.
+__device__ __forceinline__ int pf_key_tile(int64_t it, int j, int nk) { return (it & 1) ? nk - 1 - j : j; }
+
 // Persistent: each CTA walks its contiguous range of items (balanced by the host); every barrier
 // phase counts tiles over all of the CTA's items, so the producer streams the next item's K/V while
 // the current one finishes, and the O accumulator alternates between two TMEM buffers per item.
@@ -315,6 +320,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
     for (int64_t it = it0; ok && it < it1; ++it) {
       const PfItem w = pf_item(a, it);
       for (int j = 0; j < w.nk; ++j, ++g) {
+        const int kt = pf_key_tile(it, j, w.nk);
         const int st = (int)(g % NST);
         if (g >= NST && !pf_wait(&empty_bar[st], (uint32_t)((g / NST) - 1) & 1, a, &abort_flag)) {
           ok = false;
@@ -322,7 +328,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         }
         if (lane == 0) {
           mbar_expect_tx(&full_bar[st], 2 * Cf::TILE);
-          const int y = (int)(w.row_base + (int64_t)kPfRows * j);
+          const int y = (int)(w.row_base + (int64_t)kPfRows * kt);
           const uint32_t kt = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE);
 #pragma unroll
           for (int u = 0; u < Cf::NSUB; ++u) {
@@ -338,7 +344,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
 #pragma unroll
         for (int w4 = 0; w4 < 4; ++w4) {
           const int c = lane + 32 * w4;
-          const int i = kPfRows * j + c;
+          const int i = kPfRows * kt + c;
           const int hid = (i < w.ps.len ? a.meta[w.ps.moff + i] : -2) >> 1;
           none[w4] = i >= w.qr_end || hid < w.qr0;  // visible to no query of the tile
           ok_w[w4] = __ballot_sync(0xFFFFFFFFu, hid >= w.qr_end - 1);
@@ -352,7 +358,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           // per-key masking is needed when a key's visibility differs between the tile's queries,
           // or when the tile holds rows past the stored ones (their K may be anything)
           kn[st] = n_part;
-          kslow[st] = n_part > 0 || kPfRows * (j + 1) > w.ps.len || kPfRows * (j + 1) > w.qr0 + 1;
+          kslow[st] = n_part > 0 || kPfRows * (kt + 1) > w.ps.len || kPfRows * (kt + 1) > w.qr0 + 1;
         }
         // mask column of the tile: a large negative number for keys no query of the tile may see
 #pragma unroll
@@ -550,7 +556,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
 #pragma unroll
           for (int c = 0; c < CW; ++c) sv[c] = 0.f;
         }
-        const int kb = kPfRows * j;
+        const int kb = kPfRows * pf_key_tile(it, j, w.nk);
         if (kslow[st]) {
           // visibility of the tile's keys to this query as four 32-bit words: the causal prefix (key
           // row <= iq) with the tile-wide bound words plus the listed keys whose bound admits iq.
@@ -615,15 +621,22 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         const bool move = cand > m + 8.f;
         const float m_new = move ? cand : m;
         const float ref = m_new == -INFINITY ? 0.f : m_new;
-        uint32_t pk[CW / 2];
+        // P = 2^(s c2 - ref) as 16-bit pairs over the first half of this tile's S columns (row r in
+        // lane r), stored 32 columns at a time as they are made
         float2 rs4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
         const float2 c2v = make_float2(c2, c2), nref = make_float2(-ref, -ref);
+        const bool sok = __all_sync(0xFFFFFFFFu, ok);
 #pragma unroll
-        for (int c = 0; c < CW; c += 2) {
-          const float2 x = __ffma2_rn(make_float2(sv[c], sv[c + 1]), c2v, nref);
-          const float2 p = make_float2(ex2(x.x), ex2(x.y));
-          rs4[(c >> 1) & 3] = __fadd2_rn(rs4[(c >> 1) & 3], p);
-          pk[c / 2] = Pack16<T>::two(p.x, p.y);
+        for (int q = 0; q < CW / 32; ++q) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int c = 0; c < 32; c += 2) {
+            const float2 x = __ffma2_rn(make_float2(sv[32 * q + c], sv[32 * q + c + 1]), c2v, nref);
+            const float2 p = make_float2(ex2(x.x), ex2(x.y));
+            rs4[(c >> 1) & 3] = __fadd2_rn(rs4[(c >> 1) & 3], p);
+            pk[c / 2] = Pack16<T>::two(p.x, p.y);
+          }
+          if (sok) tmem_st16u(tl + sb * kPfRows + hs * (CW / 2) + 16 * q, pk);
         }
         const float rs = ((rs4[0].x + rs4[0].y) + (rs4[1].x + rs4[1].y)) + ((rs4[2].x + rs4[2].y) + (rs4[3].x + rs4[3].y));
         const float alpha = !move ? 1.f : (m == -INFINITY ? 0.f : ex2(m - ref));
@@ -648,11 +661,6 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
               tmem_st16(o_t + 16 * u, o);
             }
           }
-        }
-        // P (16-bit pairs) over the first half of this tile's S columns, row r in lane r
-        if (__all_sync(0xFFFFFFFFu, ok)) {
-#pragma unroll
-          for (int q = 0; q < CW / 32; ++q) tmem_st16u(tl + sb * kPfRows + hs * (CW / 2) + 16 * q, pk + 16 * q);
         }
         tmem_wait_st();
         if (kb + kPfRows > w.ps.len && kb + r >= w.ps.len) {
