@@ -58,3 +58,48 @@ def test_full_ragged():
     run = _full(w, 32, check_at={0, 15, 31})
     ln = run.cache.lengths()[0]
     assert ln.max() > 3000 and ln.min() < 400  # ragged: lengths span more than an order of magnitude
+
+
+# --------------------------------------------------------------------------
+# Masked prefill at the benchmark's size: the whole OPT-1.3B-shaped prompt (b = 16, L = 2048,
+# 24 layers, 32 heads), in one go and in blocks of 512 tokens, every layer prefilled as the bench
+# times it; sampled queries (block edges, <CL>/<CR> tokens, random) of three layers, three
+# sequences and two heads against the oracle's single-query attention over the mask.
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("block", [0, 512])
+def test_full_prefill_opt13b_shaped(block):
+    import oracle as orc
+
+    w = wl.opt13b()
+    layers, seqs, heads = {0, w.M // 2, w.M - 1}, [0, w.b // 2, w.b - 1], [0, w.H - 1]
+    run = harness.Runner(w, 0)
+    got = []
+
+    def keep(start, n, m, out):
+        if m in layers:
+            got.append((start.copy(), n.copy(), m, out.cpu().numpy()))
+
+    run.prefill_prompt(block=block, out_cb=keep)
+    assert run.cache.device_status() == 0
+    rng = np.random.default_rng(block + 1)
+    n_checked = 0
+    for start, n, m, o in got:
+        row0 = np.concatenate([[0], np.cumsum(n)[:-1]])
+        for s in seqs:
+            T = int(start[s] + n[s])
+            kinds = np.asarray(w.prompt_kinds[s][:T], np.uint8)
+            pos = orc.tied_positions(kinds)
+            K, V = ow.kv_bits(w, m, s, T, heads)
+            lo = int(start[s])
+            special = [t for t in range(lo, T) if kinds[t] != 0][:6]
+            ts = sorted({lo, T - 1, *special, *rng.integers(lo, T, size=8).tolist()})
+            for t in ts:
+                rows = np.nonzero(orc.visible(kinds[:t + 1], t))[0]
+                q = ow.q_bits(w, m, s, t, heads)
+                ref = np.stack([orc.attend(q[i], K[i], V[i], pos, rows, w.dtype, w.scale, w.rotary_dim, w.rope_base,
+                                           int(pos[t])) for i in range(len(heads))])
+                g = o[row0[s] + (t - lo)][heads]
+                compare(g, ref, f"prefill block={block} layer {m} seq {s} token {t}")
+                n_checked += 1
+    assert n_checked > 100
