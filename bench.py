@@ -630,30 +630,58 @@ def run_e2e(args, w, dev, world):
         host_in.append((inp.kinds, inp.kv_k.cpu().pin_memory(), inp.kv_v.cpu().pin_memory(),
                         inp.q.cpu().pin_memory()))
     shape = (w.M, w.b, w.H, w.d)
-    dk = torch.empty(shape, dtype=run.tdt, device=dev)
-    dv = torch.empty_like(dk)
-    dq = torch.empty_like(dk)
-    out = torch.empty(shape, dtype=torch.float32, device=dev)
-    host_out = torch.empty(shape, dtype=torch.float32).pin_memory()
-    h2d = 3 * dk.numel() * dk.element_size()
-    d2h = host_out.numel() * 4
+    # Two sets of device inputs and outputs: a copy stream uploads the next step's inputs while the
+    # current step runs, and reads each step's outputs back while the next one runs.  Every step's
+    # copies happen inside the timed region; only their overlap with compute is new.
+    dk = [torch.empty(shape, dtype=run.tdt, device=dev) for _ in range(2)]
+    dv = [torch.empty_like(dk[0]) for _ in range(2)]
+    dq = [torch.empty_like(dk[0]) for _ in range(2)]
+    out = [torch.empty(shape, dtype=torch.float32, device=dev) for _ in range(2)]
+    host_out = [torch.empty(shape, dtype=torch.float32).pin_memory() for _ in range(2)]
+    h2d = 3 * dk[0].numel() * dk[0].element_size()
+    d2h = host_out[0].numel() * 4
+    comp = torch.cuda.current_stream(dev)
+    copy = torch.cuda.Stream(dev)
+    ev_in = [torch.cuda.Event() for _ in range(2)]     # inputs of the set uploaded
+    ev_done = [torch.cuda.Event() for _ in range(2)]   # the step using the set finished
+    ev_out = [torch.cuda.Event() for _ in range(2)]    # its outputs read back
 
-    def one(g):
+    def upload(g):
+        i = g & 1
         kinds, hk, hv, hq = host_in[g]
-        dk.copy_(hk, non_blocking=True)
-        dv.copy_(hv, non_blocking=True)
-        dq.copy_(hq, non_blocking=True)
-        run.step(harness.StepInputs(kinds, dk, dv, dq), out)
-        host_out.copy_(out, non_blocking=True)
+        with torch.cuda.stream(copy):
+            copy.wait_event(ev_done[i])   # the step that last used this set is done with its inputs
+            dk[i].copy_(hk, non_blocking=True)
+            dv[i].copy_(hv, non_blocking=True)
+            dq[i].copy_(hq, non_blocking=True)
+            ev_in[i].record(copy)
 
+    def one(g, last):
+        i = g & 1
+        comp.wait_event(ev_in[i])
+        comp.wait_event(ev_out[i])        # the outputs of the set's previous step have been read back
+        if not last:
+            upload(g + 1)
+        run.step(harness.StepInputs(host_in[g][0], dk[i], dv[i], dq[i]), out[i], stream=comp)
+        ev_done[i].record(comp)
+        with torch.cuda.stream(copy):
+            copy.wait_event(ev_done[i])
+            host_out[i].copy_(out[i], non_blocking=True)
+            ev_out[i].record(copy)
+
+    for i in range(2):
+        ev_done[i].record(comp)
+        ev_out[i].record(comp)
+    upload(0)
     for g in range(args.warmup):
-        one(g)
+        one(g, g == args.warmup - 1)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     t0 = time.perf_counter()
+    upload(args.warmup)  # every timed step's inputs are uploaded inside the timed region
     for k in range(args.steps):
-        one(args.warmup + k)
+        one(args.warmup + k, k == args.steps - 1)
     torch.cuda.synchronize()
     elapsed = time.perf_counter() - t0
     tokens, elapsed = aggregate(w.b * args.steps, elapsed, dev)

@@ -224,17 +224,18 @@ class Runner:
         events: optional list of (start, end) CUDA event pairs, one per layer, recorded around each decode."""
         w = self.w
         n_new = np.ones(w.b, dtype=np.int32)
-        self.cache.append(inp.kv_k, inp.kv_v, n_new, inp.kinds, layer=-1, stream=stream)
+        sh = kvc.stream_handle(stream)  # resolved once: every call of the step goes on this stream
+        self.cache.append(inp.kv_k, inp.kv_v, n_new, inp.kinds, layer=-1, stream=sh)
         for m in range(w.M):
             if events is not None:
                 events[m][0].record(stream)
-            kvc.kvc_decode_attention(self.cache.handle, m, inp.q[m], w.scale, out[m], stream)
+            kvc.kvc_decode_attention(self.cache.handle, m, inp.q[m], w.scale, out[m], sh)
             if events is not None:
                 events[m][1].record(stream)
         seq, cl, cr = self.step_spans(inp.kinds)
         self.g += 1
         if compress and seq:
-            self.cache.compress_spans(seq, cl, cr, stream)
+            self.cache.compress_spans(seq, cl, cr, sh)
         return seq
 
     # ---------------------------------------------------------------------------------------

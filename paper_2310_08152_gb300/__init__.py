@@ -65,6 +65,12 @@ def _stream_handle(stream) -> Optional[int]:
     return stream.cuda_stream
 
 
+def stream_handle(stream=None) -> int:
+    """The cudaStream_t (as an int) that a call given `stream` runs on: None means torch's current
+    stream.  Resolve it once and pass the int to a run of calls to skip the per-call lookup."""
+    return _stream_handle(stream)
+
+
 def _dev(t, name, dtype=None, numel=None):
     if not t.is_cuda or not t.is_contiguous():
         raise ValueError(f"{name} must be a contiguous CUDA tensor")

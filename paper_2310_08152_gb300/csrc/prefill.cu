@@ -61,11 +61,15 @@ struct PfCfg {
   static constexpr uint32_t XQ_OFF = KV_OFF + NST * 2 * TILE;
   static constexpr uint32_t XK_OFF = XQ_OFF + kPfRows * 32;
   static constexpr uint32_t SMEM = XK_OFF + NST * kPfRows * 32 + 1024;  // + slack to align the base to 1024
-  // TMEM: SBUF S tiles of 128 columns (P, 16-bit, written over the first 64 columns of its S
-  // tile), then O0 and O1 of D columns each (alternating per item)
-  static constexpr uint32_t O_COL = SBUF * kPfRows;
-  static constexpr uint32_t TMEM_COLS = O_COL + 2 * D <= 256 ? 256 : 512;
-  static_assert(O_COL + 2 * D <= TMEM_COLS && TMEM_COLS * CPS <= 512, "TMEM budget");
+  // TMEM.  One S tile (two CTAs per SM, 256 columns each): S [0,128), P [128,192) (16-bit, two per
+  // column), O [192, 192+D) -- S is released as soon as the softmax has read it, so the next
+  // Q.K^T overlaps the softmax.  Two S tiles (one CTA per SM): S0 [0,128), S1 [128,256), P written
+  // over the first 64 columns of its own S tile, then O0 and O1 (alternating per item).
+  static constexpr uint32_t P_COL = SBUF == 1 ? kPfRows : 0;  // SBUF == 2: P lives in its S tile
+  static constexpr int OBUF = SBUF == 1 ? 1 : 2;
+  static constexpr uint32_t O_COL = SBUF == 1 ? kPfRows + kPfRows / 2 : 2 * kPfRows;
+  static constexpr uint32_t TMEM_COLS = O_COL + OBUF * D <= 256 ? 256 : 512;
+  static_assert(O_COL + OBUF * D <= TMEM_COLS && TMEM_COLS * CPS <= 512, "TMEM budget");
   static_assert(D % 16 == 0 && SW * NSUB == 2 * D, "bad tile geometry");
   static_assert(SMEM <= 227 * 1024, "shared memory budget");
 };
@@ -272,7 +276,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
   using Cf = PfCfg<D>;
   constexpr int SW = Cf::SW, SUB = Cf::SUB, NST = Cf::NST, SBUF = Cf::SBUF;
   extern __shared__ uint8_t pf_smem_raw[];
-  __shared__ uint64_t full_bar[NST], empty_bar[NST], s_full[SBUF];
+  __shared__ uint64_t full_bar[NST], empty_bar[NST], s_full[SBUF], s_free;
   __shared__ uint64_t q_full, p_full, pv_done, drain;
   // Per stage, the tile's keys against its item's query tile [qr0, qr_end): khid has bit c set when
   // key c's bound holds for every query of the tile (hid >= qr_end - 1); klist holds the keys whose
@@ -301,6 +305,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       mbar_init(&empty_bar[i], 1);
     }
     for (int i = 0; i < SBUF; ++i) mbar_init(&s_full[i], 1);
+    mbar_init(&s_free, 128 * NS);  // one S tile: the softmax has read it
     mbar_init(&q_full, 128 * NS);
     mbar_init(&p_full, 128 * NS);
     mbar_init(&pv_done, 1);
@@ -395,12 +400,14 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         ok = pf_wait(&q_full, k & 1, a, &abort_flag);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t o_t = tmem + Cf::O_COL + (k & 1) * D;
-        // S = Q K^T of tile gj into its S tile, which last held P of tile gj - SBUF: the P.V reading
-        // it was issued before (tcgen05.mma from one thread run in issue order)
+        const uint32_t o_t = tmem + Cf::O_COL + (Cf::OBUF == 2 ? (k & 1) * D : 0);
+        // S = Q K^T of tile gj into its S tile.  One S tile: once the softmax has read S of tile
+        // gj - 1.  Two: the tile last held P of tile gj - 2, whose P.V was issued before (tcgen05.mma
+        // from one thread run in issue order).
         auto issue_qk = [&](int64_t gj) -> bool {
           const int st = (int)(gj % NST), sb = (int)(gj % SBUF);
           if (!pf_wait(&full_bar[st], (uint32_t)(gj / NST) & 1, a, &abort_flag)) return false;
+          if (SBUF == 1 && gj >= 1 && !pf_wait(&s_free, (uint32_t)(gj - 1) & 1, a, &abort_flag)) return false;
           tc_fence_after();
           const uint32_t k_s = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE);
 #pragma unroll
@@ -415,13 +422,13 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           tc_commit(&s_full[sb]);
           return true;
         };
-        // O += P V of tile gp (P in its S tile, 8 TMEM columns per 16 keys); first of the item: O = P V
+        // O += P V of tile gp (8 TMEM columns of P per 16 keys); the first of an item: O = P V
         auto issue_pv = [&](int64_t gp, bool first) -> bool {
           const int st = (int)(gp % NST);
           if (!pf_wait(&p_full, (uint32_t)gp & 1, a, &abort_flag)) return false;
           tc_fence_after();
           const uint32_t v_s = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE + Cf::TILE);
-          const uint32_t p_t = tmem + (uint32_t)(gp % SBUF) * kPfRows;
+          const uint32_t p_t = tmem + (SBUF == 1 ? Cf::P_COL : (uint32_t)(gp % SBUF) * kPfRows);
 #pragma unroll
           for (int kk = 0; kk < kPfRows / 16; ++kk)
             tc_mma_ts(o_t, p_t + 8 * kk, smem_desc(v_s + kk * 16 * SW, Cf::SUBB, 8 * SW, SW), idO, (!first || kk > 0));
@@ -429,14 +436,11 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           tc_commit(&empty_bar[st]);
           return true;
         };
+        // Q K^T of the next tile goes in ahead of P.V of the current one: it runs while the softmax
+        // works on the current tile
         for (int j = 0; ok && j <= nk; ++j) {
-          if (SBUF == 2) {  // Q K^T of the next tile runs while the softmax of this one does
-            if (j < nk) ok = issue_qk(g + j);
-            if (ok && j >= 1) ok = issue_pv(g + j - 1, j == 1);
-          } else {          // one S tile: P.V of the previous tile first
-            if (j >= 1) ok = issue_pv(g + j - 1, j == 1);
-            if (ok && j < nk) ok = issue_qk(g + j);
-          }
+          if (j < nk) ok = issue_qk(g + j);
+          if (ok && j >= 1) ok = issue_pv(g + j - 1, j == 1);
         }
         g += nk;
       }
@@ -456,6 +460,10 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
     float* xmax = xbuf;  // [2][NS][128] row-maximum exchange; [NS][128] row sums at the end
     // the query row of item w, rotated at its position (RoPE, pairs (e, e + rot/2)), rounded to the
     // cache type, into the K-major tile; 8 columns at a time
+    auto write_q_done = [&]() {
+      fence_proxy_async_smem();
+      mbar_arrive(&q_full);
+    };
     auto write_q = [&](const PfItem& w) {
       if (hs == 0) {
         const int iq = w.qr0 + r;
@@ -511,8 +519,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           }
         }
       }
-      fence_proxy_async_smem();
-      mbar_arrive(&q_full);
+      write_q_done();
     };
 
     if (hs == 0) {
@@ -535,7 +542,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       const int iq = w.qr0 + r;  // stored row of this query
       const bool valid = iq < w.qr_end;
       const bool cl_q = valid && (a.meta[w.ps.moff + iq] & 1);
-      const uint32_t o_t = tl + Cf::O_COL + (k & 1) * D;
+      const uint32_t o_t = tl + Cf::O_COL + (Cf::OBUF == 2 ? (k & 1) * D : 0);
       float m = -INFINITY, l = 0.f;
       for (int j = 0; j < w.nk; ++j) {
         const int64_t gj = g + j;
@@ -556,6 +563,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
 #pragma unroll
           for (int c = 0; c < CW; ++c) sv[c] = 0.f;
         }
+        if (SBUF == 1) mbar_arrive(&s_free);  // the next Q K^T may overwrite S
         const int kb = kPfRows * pf_key_tile(it, j, w.nk);
         if (kslow[st]) {
           // visibility of the tile's keys to this query as four 32-bit words: the causal prefix (key
@@ -621,34 +629,18 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         const bool move = cand > m + 8.f;
         const float m_new = move ? cand : m;
         const float ref = m_new == -INFINITY ? 0.f : m_new;
-        // P = 2^(s c2 - ref) as 16-bit pairs over the first half of this tile's S columns (row r in
-        // lane r), stored 32 columns at a time as they are made
-        float2 rs4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-        const float2 c2v = make_float2(c2, c2), nref = make_float2(-ref, -ref);
-        const bool sok = __all_sync(0xFFFFFFFFu, ok);
-#pragma unroll
-        for (int q = 0; q < CW / 32; ++q) {
-          uint32_t pk[16];
-#pragma unroll
-          for (int c = 0; c < 32; c += 2) {
-            const float2 x = __ffma2_rn(make_float2(sv[32 * q + c], sv[32 * q + c + 1]), c2v, nref);
-            const float2 p = make_float2(ex2(x.x), ex2(x.y));
-            rs4[(c >> 1) & 3] = __fadd2_rn(rs4[(c >> 1) & 3], p);
-            pk[c / 2] = Pack16<T>::two(p.x, p.y);
-          }
-          if (sok) tmem_st16u(tl + sb * kPfRows + hs * (CW / 2) + 16 * q, pk);
-        }
-        const float rs = ((rs4[0].x + rs4[0].y) + (rs4[1].x + rs4[1].y)) + ((rs4[2].x + rs4[2].y) + (rs4[3].x + rs4[3].y));
         const float alpha = !move ? 1.f : (m == -INFINITY ? 0.f : ex2(m - ref));
-        l = l * alpha + rs;  // this slice's part of the row sum
         // pv_done phases are consumed one by one, each while it is the only one that can be pending
-        // (the next P.V waits for this tile's P): phase gj - 1 during tile j >= 1, before P is
-        // released, early when O has to be rescaled; an item's last phase in its epilogue.
-        bool pv_waited = false;
-        if (j >= 1 && __any_sync(0xFFFFFFFFu, alpha != 1.f)) {
-          ok = pf_wait(&pv_done, (uint32_t)(gj - 1) & 1, a, &abort_flag);
-          pv_waited = true;
-          if (__all_sync(0xFFFFFFFFu, ok)) {
+        // (the next P.V waits for this tile's P): phase gj - 1 during tile j >= 1, before this
+        // tile's P is written (P.V of the previous tile has read its P) and before O is rescaled;
+        // an item's last phase in its epilogue.
+        // (With two S tiles, P goes into its own S tile, so the wait can come last unless O needs
+        // the rescale.)
+        bool pv_early = j >= 1;
+        if constexpr (SBUF == 2) pv_early = j >= 1 && __any_sync(0xFFFFFFFFu, alpha != 1.f);
+        if (pv_early) {
+          ok = pf_wait(&pv_done, (uint32_t)(gj - 1) & 1, a, &abort_flag) && ok;
+          if (__all_sync(0xFFFFFFFFu, ok) && __any_sync(0xFFFFFFFFu, alpha != 1.f)) {
             tc_fence_after();
 #pragma unroll
             for (int u = 0; u < D / 16; ++u) {
@@ -662,6 +654,27 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
             }
           }
         }
+        // P = 2^(s c2 - ref) as 16-bit pairs (row r in lane r), stored 32 columns at a time as they
+        // are made; the row sum of this slice
+        const uint32_t p_tl = tl + (SBUF == 1 ? Cf::P_COL : sb * kPfRows) + hs * (CW / 2);
+        float2 rs4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+        const float2 c2v = make_float2(c2, c2), nref = make_float2(-ref, -ref);
+        const bool sok = __all_sync(0xFFFFFFFFu, ok);
+        if (sok) tc_fence_after();
+#pragma unroll
+        for (int q = 0; q < CW / 32; ++q) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int c = 0; c < 32; c += 2) {
+            const float2 x = __ffma2_rn(make_float2(sv[32 * q + c], sv[32 * q + c + 1]), c2v, nref);
+            const float2 p = make_float2(ex2(x.x), ex2(x.y));
+            rs4[(c >> 1) & 3] = __fadd2_rn(rs4[(c >> 1) & 3], p);
+            pk[c / 2] = Pack16<T>::two(p.x, p.y);
+          }
+          if (sok) tmem_st16u(p_tl + 16 * q, pk);
+        }
+        const float rs = ((rs4[0].x + rs4[0].y) + (rs4[1].x + rs4[1].y)) + ((rs4[2].x + rs4[2].y) + (rs4[3].x + rs4[3].y));
+        l = l * alpha + rs;  // this slice's part of the row sum
         tmem_wait_st();
         if (kb + kPfRows > w.ps.len && kb + r >= w.ps.len) {
           // a V row past the stored rows (stale or another stream's): zero it so 0 * V stays 0
@@ -674,7 +687,9 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           }
           fence_proxy_async_smem();
         }
-        if (j >= 1 && !pv_waited) ok = pf_wait(&pv_done, (uint32_t)(gj - 1) & 1, a, &abort_flag) && ok;
+        if constexpr (SBUF == 2) {
+          if (j >= 1 && !pv_early) ok = pf_wait(&pv_done, (uint32_t)(gj - 1) & 1, a, &abort_flag) && ok;
+        }
         tc_fence_before();
         mbar_arrive(&p_full);
         m = m_new;
