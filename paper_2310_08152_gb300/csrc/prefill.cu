@@ -194,6 +194,18 @@ struct Pack16<BF16T> {
   }
 };
 
+// 16-byte global -> shared copy that does not go through registers (src_bytes 0: zero fill).
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr) : "memory");
+  return v;
+}
+
 __device__ __forceinline__ float max3(float a, float b, float c) {
   float r;
   asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
@@ -460,66 +472,55 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
     float* xmax = xbuf;  // [2][NS][128] row-maximum exchange; [NS][128] row sums at the end
     // the query row of item w, rotated at its position (RoPE, pairs (e, e + rot/2)), rounded to the
     // cache type, into the K-major tile; 8 columns at a time
-    auto write_q_done = [&]() {
-      fence_proxy_async_smem();
-      mbar_arrive(&q_full);
+    // The query rows of item w into the K-major Q tile (row r per thread), in two halves: q_issue
+    // starts 16-byte asynchronous copies of the raw row into its swizzled slots (no registers, so
+    // they can be issued early, while the previous item's last tile is still in the softmax);
+    // q_finish waits for them, rotates the row in place for RoPE (pairs (e, e + rot/2), at the
+    // query's position, rounded to the cache type) and releases the tile to the MMA thread.
+    auto q_chunk = [&](int c8) -> uint32_t {  // shared address of 8-column chunk c8 of row r
+      const int e0 = c8 * 8;
+      const int u = e0 / SUB, cw = (e0 % SUB) / 8;
+      const int phys = cw ^ ((r * SW >> 7) & (SW / 16 - 1));
+      return smem_addr(sm + Cf::Q_OFF) + u * Cf::SUBB + r * SW + phys * 16;
     };
-    auto write_q = [&](const PfItem& w) {
+    auto q_issue = [&](const PfItem& w) {
       if (hs == 0) {
         const int iq = w.qr0 + r;
         const bool valid = iq < w.qr_end;
-        const uint32_t q_s = smem_addr(sm + Cf::Q_OFF);
         const int64_t row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : 0;
-        const uint4* src = reinterpret_cast<const uint4*>(a.q + row);
+#pragma unroll
+        for (int c8 = 0; c8 < D / 8; ++c8) cp_async16(q_chunk(c8), a.q + row + 8 * c8, valid ? 16u : 0u);
+        cp_async_commit();
+      }
+    };
+    auto q_finish = [&](const PfItem& w) {
+      if (hs == 0) {
+        cp_async_wait_all();
         const int half = a.rot / 2;
-        const int32_t qpos = (valid && half > 0) ? a.pos[a.off[w.s] + iq] : 0;
-        auto load8 = [&](int c8, float* x) {
-          if (valid) {
-            const uint4 u = __ldg(src + c8);
-            const uint32_t wd[4] = {u.x, u.y, u.z, u.w};
+        const int iq = w.qr0 + r;
+        if (half > 0 && iq < w.qr_end) {
+          const int32_t qpos = a.pos[a.off[w.s] + iq];
+          for (int c8 = 0; c8 < half / 8; ++c8) {
+            const uint32_t a1 = q_chunk(c8), a2 = q_chunk(c8 + half / 8);
+            const uint4 u1 = ld_shared_v4(a1), u2 = ld_shared_v4(a2);
+            const uint32_t w1[4] = {u1.x, u1.y, u1.z, u1.w}, w2[4] = {u2.x, u2.y, u2.z, u2.w};
+            uint32_t o1[4], o2[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-              const float2 f = T::f2(wd[e]);
-              x[2 * e] = f.x;
-              x[2 * e + 1] = f.y;
+              const float2 x1 = T::f2(w1[e]), x2 = T::f2(w2[e]);
+              float sn0, cs0, sn1, cs1;
+              rope_sincos(qpos, a.rope_g[8 * c8 + 2 * e], &sn0, &cs0);
+              rope_sincos(qpos, a.rope_g[8 * c8 + 2 * e + 1], &sn1, &cs1);
+              o1[e] = Pack16<T>::two(x1.x * cs0 - x2.x * sn0, x1.y * cs1 - x2.y * sn1);
+              o2[e] = Pack16<T>::two(x2.x * cs0 + x1.x * sn0, x2.y * cs1 + x1.y * sn1);
             }
-          } else {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) x[e] = 0.f;
-          }
-        };
-        auto store8 = [&](int c8, const float* x) {
-          const int e0 = c8 * 8;
-          const int u = e0 / SUB, cw = (e0 % SUB) / 8;
-          const int phys = cw ^ ((r * SW >> 7) & (SW / 16 - 1));
-          st_shared_v4(q_s + u * Cf::SUBB + r * SW + phys * 16, Pack16<T>::two(x[0], x[1]),
-                       Pack16<T>::two(x[2], x[3]), Pack16<T>::two(x[4], x[5]), Pack16<T>::two(x[6], x[7]));
-        };
-#pragma unroll
-        for (int c8 = 0; c8 < D / 8; ++c8) {
-          const int e0 = 8 * c8;
-          if (e0 < half) {
-            float x1[8], x2[8];
-            load8(c8, x1);
-            load8(c8 + half / 8, x2);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              float sn, cs;
-              rope_sincos(qpos, a.rope_g[e0 + e], &sn, &cs);
-              const float y1 = x1[e] * cs - x2[e] * sn;
-              x2[e] = x2[e] * cs + x1[e] * sn;
-              x1[e] = y1;
-            }
-            store8(c8, x1);
-            store8(c8 + half / 8, x2);
-          } else if (e0 >= 2 * half) {
-            float x[8];
-            load8(c8, x);
-            store8(c8, x);
+            st_shared_v4(a1, o1[0], o1[1], o1[2], o1[3]);
+            st_shared_v4(a2, o2[0], o2[1], o2[2], o2[3]);
           }
         }
       }
-      write_q_done();
+      fence_proxy_async_smem();
+      mbar_arrive(&q_full);
     };
 
     if (hs == 0) {
@@ -536,9 +537,11 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
     PfItem w{};
     if (it < it1) {
       w = pf_item(a, it);
-      write_q(w);
+      q_issue(w);
+      q_finish(w);
     }
     while (it < it1) {
+      const bool has_next = it + 1 < it1;
       const int iq = w.qr0 + r;  // stored row of this query
       const bool valid = iq < w.qr_end;
       const bool cl_q = valid && (a.meta[w.ps.moff + iq] & 1);
@@ -564,6 +567,9 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           for (int c = 0; c < CW; ++c) sv[c] = 0.f;
         }
         if (SBUF == 1) mbar_arrive(&s_free);  // the next Q K^T may overwrite S
+        // S of the item's last tile is in: every Q K^T of the item is complete, the next item's
+        // queries may go into the Q tile
+        if (has_next && j == w.nk - 1) q_issue(pf_item(a, it + 1));
         const int kb = kPfRows * pf_key_tile(it, j, w.nk);
         if (kslow[st]) {
           // visibility of the tile's keys to this query as four 32-bit words: the causal prefix (key
@@ -703,11 +709,8 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       // the next item's queries go in as soon as this item's last S tile is read (every Q K^T of
       // this item is complete), so its first tiles overlap this item's epilogue
       const int64_t next = it + 1;
-      PfItem wn{};
-      if (next < it1) {
-        wn = pf_item(a, next);
-        write_q(wn);
-      }
+      const PfItem wn = has_next ? pf_item(a, next) : w;
+      if (has_next) q_finish(wn);
       // epilogue: O / l, with l summed over the NS slices of the row
       ok = pf_wait(&pv_done, (uint32_t)(g - 1) & 1, a, &abort_flag);
       if (NS > 1) xmax[hs * kPfRows + r] = l;
