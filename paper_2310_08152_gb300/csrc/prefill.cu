@@ -48,10 +48,12 @@ struct PfCfg {
   static constexpr int NSUB = D / SUB;
   static constexpr uint32_t SUBB = kPfRows * SW;  // bytes of one subtile
   static constexpr uint32_t TILE = kPfRows * D * 2;
-  // d_head 64 runs two CTAs per SM (their softmax steps interleave), each with a single S tile in
-  // TMEM and two K/V stages; larger heads run one CTA per SM with a double-buffered S tile.
-  static constexpr int CPS = D == 64 ? 2 : 1;      // CTAs per SM
-  static constexpr int SBUF = CPS == 2 ? 1 : 2;    // S tiles in TMEM
+  // d_head 64 and 80 run two CTAs per SM (their softmax steps interleave), each with a single S
+  // tile in TMEM and two K/V stages; larger heads run one CTA per SM with a double-buffered S tile.
+  static constexpr int CPS = (D == 64 || D == 80) ? 2 : 1;  // CTAs per SM
+  static constexpr int SBUF = CPS == 2 ? 1 : 2;              // S tiles in TMEM
+  static constexpr bool PSEP = D == 64;                      // P in TMEM columns of its own
+  static constexpr bool XQT = CPS == 2 && !PSEP;             // Q's mask column in TMEM, not smem
   static constexpr int NST = CPS == 2 ? 2 : D <= 96 ? 3 : 2;  // K/V stages
   static constexpr uint32_t Q_OFF = 0;
   static constexpr uint32_t KV_OFF = TILE;
@@ -59,19 +61,23 @@ struct PfCfg {
   // stage (0 or a large negative number per key), so keys hidden from a whole query tile are masked
   // by the Q.K^T product itself.
   static constexpr uint32_t XQ_OFF = KV_OFF + NST * 2 * TILE;
-  static constexpr uint32_t XK_OFF = XQ_OFF + kPfRows * 32;
+  static constexpr uint32_t XK_OFF = XQ_OFF + (XQT ? 0 : kPfRows * 32);
   static constexpr uint32_t SMEM = XK_OFF + NST * kPfRows * 32 + 1024;  // + slack to align the base to 1024
-  // TMEM.  One S tile (two CTAs per SM, 256 columns each): S [0,128), P [128,192) (16-bit, two per
-  // column), O [192, 192+D) -- S is released as soon as the softmax has read it, so the next
-  // Q.K^T overlaps the softmax.  Two S tiles (one CTA per SM): S0 [0,128), S1 [128,256), P written
-  // over the first 64 columns of its own S tile, then O0 and O1 (alternating per item).
-  static constexpr uint32_t P_COL = SBUF == 1 ? kPfRows : 0;  // SBUF == 2: P lives in its S tile
+  // TMEM.  d_head 64 (two CTAs per SM, 256 columns each): S [0,128), P [128,192) (16-bit, two
+  // per column), O [192,256) -- S is released as soon as the softmax has read it, so the next
+  // Q.K^T overlaps the softmax.  d_head 80 (two CTAs per SM): S [0,128) with P written over its
+  // first 64 columns, O [128,208), Q's mask column [208,216) -- the next Q.K^T follows the P.V.
+  // One CTA per SM: S0 [0,128), S1 [128,256), P written over the first 64 columns of its own S
+  // tile, then O0 and O1 (alternating per item).
+  static constexpr uint32_t P_COL = PSEP ? kPfRows : 0;  // else P lives in its S tile
   static constexpr int OBUF = SBUF == 1 ? 1 : 2;
-  static constexpr uint32_t O_COL = SBUF == 1 ? kPfRows + kPfRows / 2 : 2 * kPfRows;
-  static constexpr uint32_t TMEM_COLS = O_COL + OBUF * D <= 256 ? 256 : 512;
-  static_assert(O_COL + OBUF * D <= TMEM_COLS && TMEM_COLS * CPS <= 512, "TMEM budget");
+  static constexpr uint32_t O_COL = SBUF == 2 ? 2 * kPfRows : PSEP ? kPfRows + kPfRows / 2 : kPfRows;
+  static constexpr uint32_t XQ_COL = O_COL + OBUF * D;  // with XQT: 8 columns, 16 elements per row
+  static constexpr uint32_t TMEM_END = XQ_COL + (XQT ? 8 : 0);
+  static constexpr uint32_t TMEM_COLS = TMEM_END <= 256 ? 256 : 512;
+  static_assert(TMEM_END <= TMEM_COLS && TMEM_COLS * CPS <= 512, "TMEM budget");
   static_assert(D % 16 == 0 && SW * NSUB == 2 * D, "bad tile geometry");
-  static_assert(SMEM <= 227 * 1024, "shared memory budget");
+  static_assert(SMEM <= 227 * 1024 && (CPS == 1 || SMEM + 4096 <= 113 * 1024), "shared memory budget");
 };
 
 // ---------------------------------------------------------------------------------------------
@@ -149,6 +155,11 @@ __device__ __forceinline__ void tmem_st16u(uint32_t taddr, const uint32_t* r) {
       "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
       "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
       : "memory");
+}
+__device__ __forceinline__ void tmem_st8u(uint32_t taddr, const uint32_t* r) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[0]), "r"(r[1]),
+               "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+               : "memory");
 }
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
@@ -419,7 +430,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         auto issue_qk = [&](int64_t gj) -> bool {
           const int st = (int)(gj % NST), sb = (int)(gj % SBUF);
           if (!pf_wait(&full_bar[st], (uint32_t)(gj / NST) & 1, a, &abort_flag)) return false;
-          if (SBUF == 1 && gj >= 1 && !pf_wait(&s_free, (uint32_t)(gj - 1) & 1, a, &abort_flag)) return false;
+          if (Cf::PSEP && gj >= 1 && !pf_wait(&s_free, (uint32_t)(gj - 1) & 1, a, &abort_flag)) return false;
           tc_fence_after();
           const uint32_t k_s = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE);
 #pragma unroll
@@ -429,8 +440,11 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
                    idS, kk > 0);
           }
           // + the mask column: 256 x (0 or -32768) per key
-          tc_mma(tmem + sb * kPfRows, smem_desc(xq_s, 16, 8 * 32, 32),
-                 smem_desc(xk_s + st * kPfRows * 32, 16, 8 * 32, 32), idS, 1);
+          if constexpr (Cf::XQT)
+            tc_mma_ts(tmem + sb * kPfRows, tmem + Cf::XQ_COL, smem_desc(xk_s + st * kPfRows * 32, 16, 8 * 32, 32), idS, 1);
+          else
+            tc_mma(tmem + sb * kPfRows, smem_desc(xq_s, 16, 8 * 32, 32),
+                   smem_desc(xk_s + st * kPfRows * 32, 16, 8 * 32, 32), idS, 1);
           tc_commit(&s_full[sb]);
           return true;
         };
@@ -440,7 +454,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           if (!pf_wait(&p_full, (uint32_t)gp & 1, a, &abort_flag)) return false;
           tc_fence_after();
           const uint32_t v_s = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE + Cf::TILE);
-          const uint32_t p_t = tmem + (SBUF == 1 ? Cf::P_COL : (uint32_t)(gp % SBUF) * kPfRows);
+          const uint32_t p_t = tmem + (Cf::PSEP ? Cf::P_COL : (uint32_t)(gp % SBUF) * kPfRows);
 #pragma unroll
           for (int kk = 0; kk < kPfRows / 16; ++kk)
             tc_mma_ts(o_t, p_t + 8 * kk, smem_desc(v_s + kk * 16 * SW, Cf::SUBB, 8 * SW, SW), idO, (!first || kk > 0));
@@ -451,8 +465,13 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         // Q K^T of the next tile goes in ahead of P.V of the current one: it runs while the softmax
         // works on the current tile
         for (int j = 0; ok && j <= nk; ++j) {
-          if (j < nk) ok = issue_qk(g + j);
-          if (ok && j >= 1) ok = issue_pv(g + j - 1, j == 1);
+          if (SBUF == 1 && !Cf::PSEP) {  // P sits in the one S tile: its P.V before the next Q K^T
+            if (j >= 1) ok = issue_pv(g + j - 1, j == 1);
+            if (ok && j < nk) ok = issue_qk(g + j);
+          } else {
+            if (j < nk) ok = issue_qk(g + j);
+            if (ok && j >= 1) ok = issue_pv(g + j - 1, j == 1);
+          }
         }
         g += nk;
       }
@@ -523,12 +542,22 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       mbar_arrive(&q_full);
     };
 
-    if (hs == 0) {
-      // the constant half of the mask column: 256 in column 0 of every query row
-      const uint32_t row = smem_addr(sm + Cf::XQ_OFF) + r * 32;
-      const uint32_t sw = (r >> 2) & 1;
-      st_shared_v4(row + 16 * sw, (uint32_t)T::r(256.f), 0u, 0u, 0u);
-      st_shared_v4(row + 16 * (sw ^ 1), 0u, 0u, 0u, 0u);
+    if constexpr (Cf::XQT) {
+      // the constant half of the mask column, in TMEM (row r in lane r): 256 in column 0
+      if (hs == 0) {
+        const uint32_t wd[8] = {(uint32_t)T::r(256.f), 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+        tmem_st8u(tl + Cf::XQ_COL, wd);
+        tmem_wait_st();
+      }
+      tc_fence_before();  // released to the MMA thread with the first query tile
+    } else {
+      if (hs == 0) {
+        // the constant half of the mask column: 256 in column 0 of every query row
+        const uint32_t row = smem_addr(sm + Cf::XQ_OFF) + r * 32;
+        const uint32_t sw = (r >> 2) & 1;
+        st_shared_v4(row + 16 * sw, (uint32_t)T::r(256.f), 0u, 0u, 0u);
+        st_shared_v4(row + 16 * (sw ^ 1), 0u, 0u, 0u, 0u);
+      }
     }
     bool ok = true;
     int64_t g = 0;  // tiles consumed
@@ -566,7 +595,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
 #pragma unroll
           for (int c = 0; c < CW; ++c) sv[c] = 0.f;
         }
-        if (SBUF == 1) mbar_arrive(&s_free);  // the next Q K^T may overwrite S
+        if (Cf::PSEP) mbar_arrive(&s_free);  // the next Q K^T may overwrite S
         // S of the item's last tile is in: every Q K^T of the item is complete, the next item's
         // queries may go into the Q tile
         if (has_next && j == w.nk - 1) q_issue(pf_item(a, it + 1));
@@ -662,7 +691,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         }
         // P = 2^(s c2 - ref) as 16-bit pairs (row r in lane r), stored 32 columns at a time as they
         // are made; the row sum of this slice
-        const uint32_t p_tl = tl + (SBUF == 1 ? Cf::P_COL : sb * kPfRows) + hs * (CW / 2);
+        const uint32_t p_tl = tl + (Cf::PSEP ? Cf::P_COL : sb * kPfRows) + hs * (CW / 2);
         float2 rs4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
         const float2 c2v = make_float2(c2, c2), nref = make_float2(-ref, -ref);
         const bool sok = __all_sync(0xFFFFFFFFu, ok);
