@@ -226,11 +226,13 @@ class Runner:
         n_new = np.ones(w.b, dtype=np.int32)
         sh = kvc.stream_handle(stream)  # resolved once: every call of the step goes on this stream
         self.cache.append(inp.kv_k, inp.kv_v, n_new, inp.kinds, layer=-1, stream=sh)
-        for m in range(w.M):
-            if events is not None:
+        if events is None:  # all layers in one call
+            n = w.b * w.H * w.d
+            kvc.kvc_decode_attention_layers(self.cache.handle, 0, w.M, inp.q, n, w.scale, out, n, sh)
+        else:
+            for m in range(w.M):
                 events[m][0].record(stream)
-            kvc.kvc_decode_attention(self.cache.handle, m, inp.q[m], w.scale, out[m], sh)
-            if events is not None:
+                kvc.kvc_decode_attention(self.cache.handle, m, inp.q[m], w.scale, out[m], sh)
                 events[m][1].record(stream)
         seq, cl, cr = self.step_spans(inp.kinds)
         self.g += 1

@@ -220,6 +220,15 @@ kvc_status kvc_compress_spans(kvc_cache* cache, const int32_t* seq, const int64_
  * Split-K over the kept rows with a log-sum-exp combine; reads only the kept rows. */
 kvc_status kvc_decode_attention(kvc_cache* cache, int layer, const void* q, float scale, float* out, void* stream);
 
+/* kvc_decode_attention of layers first .. first + n_layers - 1 in one call (the decode step of a
+ * model whose queries for all those layers are ready, as in the paper's throughput setting,
+ * Sec. 4.3): layer first + i reads q + i * q_layer_stride elements of the cache dtype and writes
+ * out + i * out_layer_stride floats; strides are in elements, each layer's slice laid out as for
+ * kvc_decode_attention.  The same launches as n_layers separate calls, in layer order on `stream`;
+ * on an error the layers before the failing one have been launched. */
+kvc_status kvc_decode_attention_layers(kvc_cache* cache, int first, int n_layers, const void* q, int64_t q_layer_stride,
+                                       float scale, float* out, int64_t out_layer_stride, void* stream);
+
 /* The same decode as kvc_decode_attention, for callers that cannot allocate device memory at run
  * time (for example code running inside a fixed memory pool, or under an allocator that forbids
  * new device allocations): its split-K scratch -- partial results and arrival counters -- lives in

@@ -285,6 +285,13 @@ def kvc_decode_attention(cache: int, layer: int, q, scale: float, out, stream=No
     _check(lib().kvc_decode_attention(cache, layer, _ptr(q), float(scale), _ptr(out), _stream_handle(stream)))
 
 
+def kvc_decode_attention_layers(cache: int, first: int, n_layers: int, q, q_layer_stride: int, scale: float, out,
+                                out_layer_stride: int, stream=None):
+    """kvc_decode_attention of layers [first, first + n_layers) in one call (strides in elements)."""
+    _check(lib().kvc_decode_attention_layers(cache, first, n_layers, _ptr(q), int(q_layer_stride), float(scale),
+                                             _ptr(out), int(out_layer_stride), _stream_handle(stream)))
+
+
 def kvc_decode_attention_static_scratch(cache: int, layer: int, q, scale: float, out, stream=None):
     """Decode whose split-K scratch is the library's static device array (no allocation anywhere)."""
     _check(lib().kvc_decode_attention_static_scratch(cache, layer, _ptr(q), float(scale), _ptr(out),
@@ -416,6 +423,18 @@ class KVCache:
 
     def prefill_keys(self, seq: int, n_q: int) -> np.ndarray:
         return kvc_book_prefill_keys(lib().kvc_get_book(self.handle), seq, n_q)
+
+    def decode_attention_layers(self, q, scale: float, out=None, stream=None):
+        """Decode attention of every layer in one call: q [M][b][H][d_head], out fp32 [M][b][H][d_head]."""
+        import torch
+
+        _dev(q, "q", self.torch_dtype, self.M * self.b * self.H * self.d)
+        if out is None:
+            out = torch.empty(self.M, self.b, self.H, self.d, dtype=torch.float32, device=q.device)
+        _dev(out, "out", torch.float32, self.M * self.b * self.H * self.d)
+        n = self.b * self.H * self.d
+        kvc_decode_attention_layers(self.handle, 0, self.M, q, n, scale, out, n, stream)
+        return out
 
     def masked_reference_layout(self, seq: int, stream=None):
         cap = _layout_sizes(lib().kvc_book_layout, lib().kvc_get_book(self.handle), seq)

@@ -57,6 +57,7 @@ SIGNATURES = [
     ("kvc_compress_spans", c_int, [P, P, P, P, c_int, P]),
     ("kvc_decode_attention", c_int, [P, c_int, P, c_float, P, P]),
     ("kvc_decode_attention_static_scratch", c_int, [P, c_int, P, c_float, P, P]),
+    ("kvc_decode_attention_layers", c_int, [P, c_int, c_int, P, c_int64, c_float, P, c_int64, P]),
     ("kvc_prefill_attention", c_int, [P, c_int, P, P, c_float, P, P]),
     ("kvc_masked_reference_layout", c_int, [P, c_int, c_int64, P, P, P, P, P, P, P, P]),
     ("kvc_device_status", c_int, [P, P, P]),

@@ -779,6 +779,24 @@ kvc_status kvc_decode_attention(kvc_cache* c, int layer, const void* q, float sc
   return ok();
 }
 
+kvc_status kvc_decode_attention_layers(kvc_cache* c, int first, int n_layers, const void* q, int64_t q_layer_stride,
+                                       float scale, float* out, int64_t out_layer_stride, void* stream) {
+  if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
+  if (n_layers < 0 || first < 0 || first + n_layers > c->cfg.M)
+    return fail(KVC_ERR_INVALID_ARG, "layers [%d, %d) out of range [0, %d)", first, first + n_layers, c->cfg.M);
+  if (n_layers > 0 && (!q || !out)) return fail(KVC_ERR_INVALID_ARG, "q/out are NULL");
+  const int64_t need = (int64_t)c->cfg.b * c->cfg.H * c->cfg.d_head;
+  if (n_layers > 1 && (q_layer_stride < need || out_layer_stride < need))
+    return fail(KVC_ERR_INVALID_ARG, "layer strides (%lld, %lld) below one layer's %lld elements",
+                (long long)q_layer_stride, (long long)out_layer_stride, (long long)need);
+  const uint16_t* qp = static_cast<const uint16_t*>(q);
+  for (int i = 0; i < n_layers; ++i) {
+    kvc_status st = kvc_decode_attention(c, first + i, qp + i * q_layer_stride, scale, out + i * out_layer_stride, stream);
+    if (st != KVC_OK) return st;
+  }
+  return ok();
+}
+
 kvc_status kvc_decode_attention_static_scratch(kvc_cache* c, int layer, const void* q, float scale, float* out,
                                                void* stream_) {
   if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");

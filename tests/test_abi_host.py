@@ -219,6 +219,11 @@ def test_cache_validates_before_any_device_work():
         assert L.kvc_append(h, 1, fake, fake, None, None, None, None) == 5   # layer 1 before layer 0
         assert L.kvc_decode_attention(h, 0, fake, ctypes.c_float(0.125), fake, None) == 5  # nothing appended
         assert L.kvc_decode_attention(h, 9, fake, ctypes.c_float(0.125), fake, None) == 1
+        n = 2 * 4 * 64
+        assert L.kvc_decode_attention_layers(h, 1, 2, fake, n, ctypes.c_float(0.125), fake, n, None) == 1  # > M
+        assert L.kvc_decode_attention_layers(h, 0, 2, fake, n - 1, ctypes.c_float(0.125), fake, n, None) == 1
+        assert L.kvc_decode_attention_layers(h, 0, 2, fake, n, ctypes.c_float(0.125), fake, n, None) == 5
+        assert L.kvc_decode_attention_layers(h, 0, 0, None, 0, ctypes.c_float(0.125), None, 0, None) == 0
         assert L.kvc_compress_spans(h, np.int32([0]).ctypes.data, np.int64([0]).ctypes.data,
                                     np.int64([1]).ctypes.data, 1, None) == 4
         assert b"span" in L.kvc_last_error() or b"closed" in L.kvc_last_error()

@@ -286,3 +286,28 @@ def test_local_attention_fifo_cache(ratio):
                 first = int(np.floor(T * np.float64(r32)))
                 assert np.array_equal(lay["stored_orig"], np.arange(first, T))
         assert run.cache.device_status() == 0
+
+
+def test_multi_layer_decode_call_equals_per_layer_calls():
+    """kvc_decode_attention_layers launches exactly the per-layer decodes: identical outputs."""
+    w = wl.opt13b(b=3, L=400, M=3)
+    run = harness.Runner(w, 2)
+    run.load_prompt()
+    inp = run.make_step_inputs(0)
+    run.cache.append(inp.kv_k, inp.kv_v, np.ones(w.b, np.int32), inp.kinds)
+    one = torch.full((w.M, w.b, w.H, w.d), float("nan"), dtype=torch.float32, device="cuda")
+    for m in range(w.M):
+        kvc.kvc_decode_attention(run.cache.handle, m, inp.q[m], w.scale, one[m])
+    many = run.cache.decode_attention_layers(inp.q, w.scale)
+    torch.cuda.synchronize()
+    assert torch.equal(one, many)
+    # a run of layers in the middle, with padded strides
+    n = w.b * w.H * w.d
+    qpad = torch.zeros(w.M, n + 64, dtype=inp.q.dtype, device="cuda")
+    qpad[:, :n] = inp.q.reshape(w.M, n)
+    opad = torch.full((w.M, n + 32), float("nan"), dtype=torch.float32, device="cuda")
+    kvc.kvc_decode_attention_layers(run.cache.handle, 1, 2, qpad[1], n + 64, w.scale, opad[1], n + 32)
+    torch.cuda.synchronize()
+    assert torch.equal(opad[1:, :n], one[1:].reshape(2, n))
+    assert torch.isnan(opad[0]).all()
+    assert run.cache.device_status() == 0
