@@ -648,9 +648,17 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           for (int u = 0; u < 8; ++u) mx8[u] = fmaxf(mx8[u], sv[CW - 8 + u]);
         }
         float mx = max3(max3(mx8[0], mx8[1], mx8[2]), max3(mx8[3], mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]));
-        if (NS > 1) xmax[((gj & 1) * NS + hs) * kPfRows + r] = mx;
-        // every softmax thread passes this barrier: the exit decision is taken by all of them at once
-        if (!bar_and(1, NSM, ok)) {
+        if (NS > 1) {
+          xmax[((gj & 1) * NS + hs) * kPfRows + r] = mx;
+          // every softmax thread passes this barrier: the exit decision is taken by all of them at once
+          if (!bar_and(1, NSM, ok)) {
+            ok = false;
+            break;
+          }
+        } else if (!__all_sync(0xFFFFFFFFu, ok)) {
+          // one slice per row: no exchange, so no barrier inside the tile loop -- a warp that stops
+          // here meets the others at the barrier after the loop (their bounded waits give up at once
+          // once any role has given up)
           ok = false;
           break;
         }
