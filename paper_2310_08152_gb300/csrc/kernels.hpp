@@ -102,18 +102,25 @@ cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& bu
 struct PState {
   int32_t len, q0, qtok, moff;
 };
+// One prefill work item (sequence s, head h, query tile [qr0, qr_end)) as the host lays it out,
+// in the kernel's order; row0 = seq_row0[s] + h * cap[s], the K/V plane row of stored row 0 in
+// layer 0 (the kernel adds layer * H * C).
+struct PfItemRec {
+  PState ps;
+  int32_t s, h, qr0, qr_end;
+  int32_t nk, row0_lo, row0_hi, pad;
+};
+static_assert(sizeof(PfItemRec) == 48, "three 16-byte loads");
 
 struct PrefillArgs {
   int layer, H, b, rot;
   int64_t C;
-  const PState* ps;        // [b]
-  const int32_t* Pq;       // [b+1] prefix sums of query tiles (128 queries each)
-  int64_t n_items;         // H * Pq[b]: (query tile, head) work items
+  const PfItemRec* items;  // [n_items], sequence-major, then head, then the query tile with the most keys first
+  int64_t n_items;         // (query tile, head) work items
   const int32_t* cta_items; // [n_ctas + 1]: CTA c takes items [cta_items[c], cta_items[c+1])
   int n_ctas;              // persistent grid size
   const int32_t* meta;     // per stored row: (hid << 1) | is_cl
   const uint16_t* q;       // [sum n_q][H][D]
-  const uint16_t* v;       // cache V planes (a <CL> query's output is its own value row)
   float* out;              // [sum n_q][H][D]
   float c2;                // scale * log2(e)
   const int32_t* pos;      // [C] stored-row positions

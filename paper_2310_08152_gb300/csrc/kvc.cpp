@@ -58,9 +58,10 @@ struct WsLayout {
   size_t src_map = 0;    // int32 [C]: source row of each destination row of a compaction
   size_t counters = 0;   // int32 [b*H]
   size_t partials = 0;   // float [(kMaxDecodeWorkers + b*H) * (D + 4)]
-  size_t pre = 0;        // prefill plan: [PState b][int32 Pq b+1][int32 meta C]
-  size_t pre_Pq = 0;     // offsets inside the prefill plan
-  size_t pre_cta = 0;     // int32 [kMaxPrefillCtas + 1]: each CTA's range of work items
+  size_t pre = 0;        // prefill plan: [int32 cta][PfItemRec items][int32 meta C]
+  size_t pre_cta = 0;    // offsets inside the plan; int32 [kMaxPrefillCtas + 1]: each CTA's item range
+  size_t pre_items = 0;  // PfItemRec [pre_max_items]
+  int64_t pre_max_items = 0;
   size_t pre_meta = 0;
   size_t pre_bytes = 0;
   size_t total = 0;
@@ -88,9 +89,12 @@ WsLayout ws_layout(int b, int H, int D, int rot, int64_t C) {
   L.src_map = take(4 * (size_t)C);
   L.counters = take(4 * (size_t)b * H);
   L.partials = take(4 * (size_t)(kvc::kMaxDecodeWorkers + (int64_t)b * H) * (size_t)(D + 4));
-  L.pre_Pq = align_up(sizeof(kvc::PState) * (size_t)b, 16);
-  L.pre_cta = align_up(L.pre_Pq + 4 * (size_t)(b + 1), 16);
-  L.pre_meta = align_up(L.pre_cta + 4 * (size_t)(kvc::kMaxPrefillCtas + 1), 16);
+  // work items: H per query tile, and a sequence of capacity cap has at most ceil(cap / 128) query
+  // tiles, so at most H * (C / 128 + b) in all
+  L.pre_cta = 0;
+  L.pre_items = align_up(4 * (size_t)(kvc::kMaxPrefillCtas + 1), 16);
+  L.pre_max_items = (int64_t)H * ((C + 127) / 128 + b);
+  L.pre_meta = align_up(L.pre_items + sizeof(kvc::PfItemRec) * (size_t)L.pre_max_items, 16);
   L.pre_bytes = L.pre_meta + 4 * (size_t)C;
   L.pre = take(L.pre_bytes);
   L.total = o;
@@ -889,8 +893,8 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
     const size_t bytes = c->ws.pre_meta + 4 * n_meta;
     unsigned char* img = c->ring.reserve(bytes, &e);
     if (!img) return e != cudaSuccess ? cuda_fail(e, "staging") : fail(KVC_ERR_INVALID_ARG, "prefill plan exceeds ring");
-    kvc::PState* ps = reinterpret_cast<kvc::PState*>(img);
-    int32_t* Pq = reinterpret_cast<int32_t*>(img + c->ws.pre_Pq);
+    std::vector<kvc::PState> ps(b);
+    std::vector<int32_t> Pq(b + 1);
     int32_t* meta = reinterpret_cast<int32_t*>(img + c->ws.pre_meta);
     int64_t qtok = 0, moff = 0;
     Pq[0] = 0;
@@ -910,6 +914,7 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
     // one per CTA of the persistent grid: balanced, and each CTA stays on a few (sequence, head)
     // streams whose K/V rows it re-reads from L2.
     const int64_t n_items = (int64_t)H * Pq[b];
+    if (n_items > c->ws.pre_max_items) return fail(KVC_ERR_INVALID_ARG, "prefill work items exceed the plan");
     const int G = (int)std::min<int64_t>(
         std::min(c->num_sms * kvc::prefill_ctas_per_sm(c->cfg.d_head), kvc::kMaxPrefillCtas), n_items);
     int32_t* cta = reinterpret_cast<int32_t*>(img + c->ws.pre_cta);
@@ -926,6 +931,7 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
     }
     cta[0] = 0;
     {
+      kvc::PfItemRec* items = reinterpret_cast<kvc::PfItemRec*>(img + c->ws.pre_items);
       int c_next = 1;
       double acc = 0.0;
       int64_t item = 0;
@@ -936,6 +942,18 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
           for (int k = 0; k < nqt; ++k, ++item) {
             acc += work_sq[base + k];
             while (c_next < G && acc >= W * c_next / G) cta[c_next++] = (int32_t)(item + 1);
+            kvc::PfItemRec& r = items[item];
+            const int qt = nqt - 1 - k;
+            r.ps = ps[s];
+            r.s = s;
+            r.h = h;
+            r.qr0 = ps[s].q0 + 128 * qt;
+            r.qr_end = std::min(r.qr0 + 128, ps[s].len);
+            r.nk = (r.qr_end + 127) / 128;
+            const int64_t row0 = (int64_t)H * c->off[s] + (int64_t)h * c->cap[s];  // = seq_row0[s] + h * cap[s]
+            r.row0_lo = (int32_t)(uint32_t)(uint64_t)row0;
+            r.row0_hi = (int32_t)((uint64_t)row0 >> 32);
+            r.pad = 0;
           }
         base += nqt;
       }
@@ -955,11 +973,9 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
   a.b = b;
   a.rot = c->cfg.rotary_dim;
   a.C = c->C;
-  a.ps = reinterpret_cast<const kvc::PState*>(c->wsp(c->ws.pre));
-  a.Pq = reinterpret_cast<const int32_t*>(c->wsp(c->ws.pre + c->ws.pre_Pq));
+  a.items = reinterpret_cast<const kvc::PfItemRec*>(c->wsp(c->ws.pre + c->ws.pre_items));
   a.meta = reinterpret_cast<const int32_t*>(c->wsp(c->ws.pre + c->ws.pre_meta));
   a.q = static_cast<const uint16_t*>(q);
-  a.v = static_cast<const uint16_t*>(c->cfg.v_base);
   a.out = out;
   a.c2 = (float)((double)scale * 1.4426950408889634);
   a.pos = c->cfg.pos_base;

@@ -209,6 +209,9 @@ struct Pack16<BF16T> {
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
 }
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
@@ -216,6 +219,9 @@ __device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
   asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr) : "memory");
   return v;
 }
+
+// Bits [0, n) of a 32-bit word, n clamped to [0, 32].
+__device__ __forceinline__ uint32_t low_bits(int n) { return n <= 0 ? 0u : n >= 32 ? 0xFFFFFFFFu : (1u << n) - 1u; }
 
 __device__ __forceinline__ float max3(float a, float b, float c) {
   float r;
@@ -253,8 +259,7 @@ __device__ __forceinline__ bool pf_wait(uint64_t* bar, uint32_t parity, const Pr
   }
 }
 
-// One work item: query tile qt of (sequence s, head h).  Items of sequence s are
-// [H * Pq[s], H * Pq[s+1]), head-major, the tile with the most keys first.
+// One work item: query tile [qr0, qr_end) of (sequence s, head h), read from the host's table.
 struct PfItem {
   PState ps;
   int s, h, qr0, qr_end, nk;
@@ -262,25 +267,16 @@ struct PfItem {
 };
 
 __device__ __forceinline__ PfItem pf_item(const PrefillArgs& a, int64_t it) {
-  int lo = 0, hi = a.b - 1;  // last s with H * Pq[s] <= it
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if ((int64_t)a.H * a.Pq[mid] <= it)
-      lo = mid;
-    else
-      hi = mid - 1;
-  }
+  const int4* r = reinterpret_cast<const int4*>(a.items + it);
+  const int4 x = __ldg(r), y = __ldg(r + 1), z = __ldg(r + 2);
   PfItem w;
-  const int nqt = a.Pq[lo + 1] - a.Pq[lo];
-  const int64_t local = it - (int64_t)a.H * a.Pq[lo];
-  w.ps = a.ps[lo];
-  w.s = lo;
-  w.h = (int)(local / nqt);
-  const int qt = nqt - 1 - (int)(local % nqt);
-  w.qr0 = w.ps.q0 + kPfRows * qt;                   // first query row of the tile
-  w.qr_end = min(w.qr0 + kPfRows, w.ps.len);        // one past its last
-  w.nk = (w.qr_end + kPfRows - 1) / kPfRows;        // key tiles [0, nk)
-  w.row_base = (int64_t)a.layer * a.H * a.C + a.seq_row0[lo] + (int64_t)w.h * a.cap[lo];
+  w.ps = PState{x.x, x.y, x.z, x.w};
+  w.s = y.x;
+  w.h = y.y;
+  w.qr0 = y.z;
+  w.qr_end = y.w;
+  w.nk = z.x;
+  w.row_base = (int64_t)a.layer * a.H * a.C + (int64_t)(((uint64_t)(uint32_t)z.z << 32) | (uint32_t)z.y);
   return w;
 }
 
@@ -302,13 +298,18 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
   __shared__ uint64_t full_bar[NST], empty_bar[NST], s_full[SBUF], s_free;
   __shared__ uint64_t q_full, p_full, pv_done, drain;
   // Per stage, the tile's keys against its item's query tile [qr0, qr_end): khid has bit c set when
-  // key c's bound holds for every query of the tile (hid >= qr_end - 1); klist holds the keys whose
-  // bound falls inside it (qr0 <= hid < qr_end - 1: a span closing among the queries), kn of them.
+  // key c's bound holds for every query of the tile (hid >= qr_end - 1).  The keys whose bound falls
+  // inside it (qr0 <= hid < qr_end - 1: a span closing among the queries) come in runs of one bound
+  // -- a span's interior shares its <CR>, a <CL> hidden from every later query is a run of one --
+  // kept as the bound (rhid) and the column range [cb, ce) (rcol = cb | ce << 16), kn runs.
   __shared__ uint4 khid[NST];
-  __shared__ int2 klist[NST][kPfRows];
+  __shared__ int32_t rhid[NST][kPfRows];
+  __shared__ uint32_t rcol[NST][kPfRows];
   __shared__ int32_t kn[NST];
-  __shared__ int32_t kslow[NST];  // the tile needs the per-key rule (else its mask column decides)
-  __shared__ float xbuf[2 * NS * kPfRows];
+  __shared__ int32_t kslow[NST];  // the tile needs the per-key rule (else its mask columns decide)
+  __shared__ float xbuf[NS > 1 ? 2 * NS * kPfRows : 1];
+  __shared__ PfItem next_item;  // the item after the current one, as the softmax warps found it
+  __shared__ int32_t qmeta[kPfRows];  // mask bounds of the query rows of the next item
   __shared__ uint32_t tmem_slot;
   __shared__ volatile int abort_flag;
 
@@ -368,7 +369,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         // sorted into the classes above; the causal part (i <= iq) is left to each query
         uint32_t ok_w[4];
         bool none[4];
-        int n_part = 0;
+        int hp[4];  // the key's bound when it falls among the queries, else -3
 #pragma unroll
         for (int w4 = 0; w4 < 4; ++w4) {
           const int c = lane + 32 * w4;
@@ -376,26 +377,49 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           const int hid = (i < w.ps.len ? a.meta[w.ps.moff + i] : -2) >> 1;
           none[w4] = i >= w.qr_end || hid < w.qr0;  // visible to no query of the tile
           ok_w[w4] = __ballot_sync(0xFFFFFFFFu, hid >= w.qr_end - 1);
-          const bool part = hid >= w.qr0 && hid < w.qr_end - 1;
-          const uint32_t pb = __ballot_sync(0xFFFFFFFFu, part);
-          if (part) klist[st][n_part + __popc(pb & ((1u << lane) - 1u))] = make_int2(c, hid);
-          n_part += __popc(pb);
+          hp[w4] = hid >= w.qr0 && hid < w.qr_end - 1 ? hid : -3;
         }
-        if (lane == 0) {
-          khid[st] = make_uint4(ok_w[0], ok_w[1], ok_w[2], ok_w[3]);
-          // per-key masking is needed when a key's visibility differs between the tile's queries,
-          // or when the tile holds rows past the stored ones (their K may be anything)
-          kn[st] = n_part;
-          kslow[st] = n_part > 0 || kPfRows * (kt + 1) > w.ps.len || kPfRows * (kt + 1) > w.qr0 + 1;
-        }
-        // mask column of the tile: a large negative number for keys no query of the tile may see
+        // runs: a listed key starts one unless key c - 1 is listed with the same bound, and ends one
+        // unless key c + 1 is
+        int n_run = 0;
 #pragma unroll
         for (int w4 = 0; w4 < 4; ++w4) {
           const int c = lane + 32 * w4;
-          const uint32_t x0 = none[w4] ? (uint32_t)T::r(-32768.f) : 0u;
+          int prev = __shfl_up_sync(0xFFFFFFFFu, hp[w4], 1);
+          int next = __shfl_down_sync(0xFFFFFFFFu, hp[w4], 1);
+          const int prev_w = w4 > 0 ? __shfl_sync(0xFFFFFFFFu, hp[w4 > 0 ? w4 - 1 : 0], 31) : -3;
+          const int next_w = w4 < 3 ? __shfl_sync(0xFFFFFFFFu, hp[w4 < 3 ? w4 + 1 : 3], 0) : -3;
+          if (lane == 0) prev = prev_w;
+          if (lane == 31) next = next_w;
+          const bool start = hp[w4] >= 0 && prev != hp[w4];
+          const bool end = hp[w4] >= 0 && next != hp[w4];
+          const uint32_t sb = __ballot_sync(0xFFFFFFFFu, start);
+          const int rid = n_run + __popc(sb & ((2u << lane) - 1u)) - 1;  // runs started at or before c, less one
+          if (start) {
+            rhid[st][rid] = hp[w4];
+            reinterpret_cast<uint16_t*>(&rcol[st][rid])[0] = (uint16_t)c;
+          }
+          if (end) reinterpret_cast<uint16_t*>(&rcol[st][rid])[1] = (uint16_t)(c + 1);
+          n_run += __popc(sb);
+        }
+        if (lane == 0) {
+          khid[st] = make_uint4(ok_w[0], ok_w[1], ok_w[2], ok_w[3]);
+          // per-key masking is needed when a key's visibility differs between the tile's queries
+          // (runs; keys at or past the first query: the causal rule, and a <CL> query sees only
+          // itself), or when the tile holds rows past the stored ones (their K may be anything)
+          kn[st] = n_run;
+          kslow[st] = n_run > 0 || kPfRows * (kt + 1) > w.ps.len || kPfRows * (kt + 1) > w.qr0;
+        }
+        // mask columns of the tile, 0 or a large negative number per key: column 0 for keys no query
+        // of the tile may see, column 1 for keys before the query tile (a <CL> query sees only itself)
+#pragma unroll
+        for (int w4 = 0; w4 < 4; ++w4) {
+          const int c = lane + 32 * w4;
+          const uint32_t neg = (uint32_t)T::r(-32768.f);
+          const uint32_t x01 = (none[w4] ? neg : 0u) | (kPfRows * kt + c < w.qr0 ? neg << 16 : 0u);
           const uint32_t row = smem_addr(sm + Cf::XK_OFF + st * kPfRows * 32) + c * 32;
           const uint32_t sw = (c >> 2) & 1;  // 32-byte swizzle: the two 16-byte halves swap every 4 rows
-          st_shared_v4(row + 16 * sw, x0, 0u, 0u, 0u);
+          st_shared_v4(row + 16 * sw, x01, 0u, 0u, 0u);
           st_shared_v4(row + 16 * (sw ^ 1), 0u, 0u, 0u, 0u);
         }
         fence_proxy_async_smem();
@@ -495,7 +519,9 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
     // starts 16-byte asynchronous copies of the raw row into its swizzled slots (no registers, so
     // they can be issued early, while the previous item's last tile is still in the softmax);
     // q_finish waits for them, rotates the row in place for RoPE (pairs (e, e + rot/2), at the
-    // query's position, rounded to the cache type) and releases the tile to the MMA thread.
+    // query's position, rounded to the cache type), writes the row's mask columns (256 in column 0;
+    // 256 in column 1 for a <CL> query, which the keys before the query tile then mask) and
+    // releases the tile to the MMA thread.
     auto q_chunk = [&](int c8) -> uint32_t {  // shared address of 8-column chunk c8 of row r
       const int e0 = c8 * 8;
       const int u = e0 / SUB, cw = (e0 % SUB) / 8;
@@ -509,6 +535,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         const int64_t row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : 0;
 #pragma unroll
         for (int c8 = 0; c8 < D / 8; ++c8) cp_async16(q_chunk(c8), a.q + row + 8 * c8, valid ? 16u : 0u);
+        cp_async4(smem_addr(&qmeta[r]), a.meta + (valid ? w.ps.moff + iq : 0), valid ? 4u : 0u);
         cp_async_commit();
       }
     };
@@ -537,28 +564,23 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
             st_shared_v4(a2, o2[0], o2[1], o2[2], o2[3]);
           }
         }
+        const uint32_t x01 = (uint32_t)T::r(256.f) | (qmeta[r] & 1 ? (uint32_t)T::r(256.f) << 16 : 0u);
+        if constexpr (Cf::XQT) {
+          const uint32_t wd[8] = {x01, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+          tmem_st8u(tl + Cf::XQ_COL, wd);
+          tmem_wait_st();
+          tc_fence_before();
+        } else {
+          const uint32_t row = smem_addr(sm + Cf::XQ_OFF) + r * 32;
+          const uint32_t sw = (r >> 2) & 1;  // 32-byte swizzle: the two 16-byte halves swap every 4 rows
+          st_shared_v4(row + 16 * sw, x01, 0u, 0u, 0u);
+          st_shared_v4(row + 16 * (sw ^ 1), 0u, 0u, 0u, 0u);
+        }
       }
       fence_proxy_async_smem();
       mbar_arrive(&q_full);
     };
 
-    if constexpr (Cf::XQT) {
-      // the constant half of the mask column, in TMEM (row r in lane r): 256 in column 0
-      if (hs == 0) {
-        const uint32_t wd[8] = {(uint32_t)T::r(256.f), 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-        tmem_st8u(tl + Cf::XQ_COL, wd);
-        tmem_wait_st();
-      }
-      tc_fence_before();  // released to the MMA thread with the first query tile
-    } else {
-      if (hs == 0) {
-        // the constant half of the mask column: 256 in column 0 of every query row
-        const uint32_t row = smem_addr(sm + Cf::XQ_OFF) + r * 32;
-        const uint32_t sw = (r >> 2) & 1;
-        st_shared_v4(row + 16 * sw, (uint32_t)T::r(256.f), 0u, 0u, 0u);
-        st_shared_v4(row + 16 * (sw ^ 1), 0u, 0u, 0u, 0u);
-      }
-    }
     bool ok = true;
     int64_t g = 0;  // tiles consumed
     uint32_t k = 0;  // items done
@@ -568,12 +590,13 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       w = pf_item(a, it);
       q_issue(w);
       q_finish(w);
+      if (NS > 1) bar_and(1, NSM, true);  // qmeta is read by every slice of the row
     }
     while (it < it1) {
       const bool has_next = it + 1 < it1;
       const int iq = w.qr0 + r;  // stored row of this query
       const bool valid = iq < w.qr_end;
-      const bool cl_q = valid && (a.meta[w.ps.moff + iq] & 1);
+      const bool cl_q = valid && (qmeta[r] & 1);
       const uint32_t o_t = tl + Cf::O_COL + (Cf::OBUF == 2 ? (k & 1) * D : 0);
       float m = -INFINITY, l = 0.f;
       for (int j = 0; j < w.nk; ++j) {
@@ -598,33 +621,36 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         if (Cf::PSEP) mbar_arrive(&s_free);  // the next Q K^T may overwrite S
         // S of the item's last tile is in: every Q K^T of the item is complete, the next item's
         // queries may go into the Q tile
-        if (has_next && j == w.nk - 1) q_issue(pf_item(a, it + 1));
+        if (has_next && j == w.nk - 1) {
+          const PfItem nx = pf_item(a, it + 1);
+          q_issue(nx);
+          if (lane == 0) next_item = nx;  // every warp writes the same item
+        }
         const int kb = kPfRows * pf_key_tile(it, j, w.nk);
         if (kslow[st]) {
           // visibility of the tile's keys to this query as four 32-bit words: the causal prefix (key
-          // row <= iq) with the tile-wide bound words plus the listed keys whose bound admits iq.
-          // (<CL> queries take their own value row in the epilogue.)  Other tiles are masked by
-          // their mask column alone.
+          // row <= iq) with the tile-wide bound words plus the runs whose bound admits iq.  Other
+          // tiles are masked by their mask columns alone.
           const int t = iq - kb;  // last visible column
-          auto prefix = [t](int wd) -> uint32_t {
-            const int n = t - 32 * wd + 1;  // columns of word wd at or before t
-            return n <= 0 ? 0u : n >= 32 ? 0xFFFFFFFFu : (1u << n) - 1u;
-          };
           const uint4 hw = khid[st];
           uint32_t v0 = hw.x, v1 = hw.y, v2 = hw.z, v3 = hw.w;
-          const int np = kn[st];
-          for (int e = 0; e < np; ++e) {
-            const int2 ent = klist[st][e];
-            if (ent.y >= iq) {
-              const uint32_t bit = 1u << (ent.x & 31);
-              const int wd = ent.x >> 5;
-              v0 |= wd == 0 ? bit : 0u;
-              v1 |= wd == 1 ? bit : 0u;
-              v2 |= wd == 2 ? bit : 0u;
-              v3 |= wd == 3 ? bit : 0u;
+          const int nr = kn[st];
+          for (int e = 0; e < nr; ++e) {
+            if (rhid[st][e] >= iq) {
+              const uint32_t cc = rcol[st][e];
+              const int cb = (int)(cc & 0xFFFFu), ce = (int)(cc >> 16);
+              v0 |= low_bits(ce) & ~low_bits(cb);
+              v1 |= low_bits(ce - 32) & ~low_bits(cb - 32);
+              v2 |= low_bits(ce - 64) & ~low_bits(cb - 64);
+              v3 |= low_bits(ce - 96) & ~low_bits(cb - 96);
             }
           }
-          v0 &= prefix(0), v1 &= prefix(1), v2 &= prefix(2), v3 &= prefix(3);
+          // the causal prefix; a <CL> query sees its own key alone
+          const int t1 = t + 1, t0 = cl_q ? t : 0;
+          v0 &= low_bits(t1) & ~low_bits(t0);
+          v1 &= low_bits(t1 - 32) & ~low_bits(t0 - 32);
+          v2 &= low_bits(t1 - 64) & ~low_bits(t0 - 64);
+          v3 &= low_bits(t1 - 96) & ~low_bits(t0 - 96);
           // this thread's words: columns [hs * CW, hs * CW + CW)
           uint32_t vw[CW / 32];
 #pragma unroll
@@ -635,17 +661,20 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
 #pragma unroll
           for (int c = 0; c < CW; ++c) sv[c] = (vw[c >> 5] >> (c & 31)) & 1u ? sv[c] : -INFINITY;
         }
-        // row max: a tree over this slice, then across the NS slices of the row
+        // row max: a tree over this slice (eight partial maxima: columns 0-7, then pairs of 8-column
+        // blocks, then the last block when one is left over), then across the NS slices of the row
+        static_assert(CW % 8 == 0, "slice width");
+        constexpr int kPairEnd = 8 + (CW - 8) / 16 * 16;  // columns [8, kPairEnd) go in pairs of blocks
         float mx8[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) mx8[u] = sv[u];
 #pragma unroll
-        for (int c = 8; c + 16 <= CW; c += 16)
+        for (int c = 8; c < kPairEnd; c += 16)
 #pragma unroll
           for (int u = 0; u < 8; ++u) mx8[u] = max3(mx8[u], sv[c + u], sv[c + 8 + u]);
-        if (CW % 16 == 8) {
+        if constexpr (kPairEnd < CW) {
 #pragma unroll
-          for (int u = 0; u < 8; ++u) mx8[u] = fmaxf(mx8[u], sv[CW - 8 + u]);
+          for (int u = 0; u < 8; ++u) mx8[u] = fmaxf(mx8[u], sv[kPairEnd + u]);
         }
         float mx = max3(max3(mx8[0], mx8[1], mx8[2]), max3(mx8[3], mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]));
         if (NS > 1) {
@@ -746,7 +775,8 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       // the next item's queries go in as soon as this item's last S tile is read (every Q K^T of
       // this item is complete), so its first tiles overlap this item's epilogue
       const int64_t next = it + 1;
-      const PfItem wn = has_next ? pf_item(a, next) : w;
+      __syncwarp();
+      const PfItem wn = has_next ? next_item : w;
       if (has_next) q_finish(wn);
       // epilogue: O / l, with l summed over the NS slices of the row
       ok = pf_wait(&pv_done, (uint32_t)(g - 1) & 1, a, &abort_flag);
@@ -763,31 +793,47 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       }
       tc_fence_after();
       const float inv = 1.f / lt;
-      const int64_t out_row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : 0;
+      const int64_t out_row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : -1;
+      // O / l to global memory.  Each group of four lanes (four consecutive query rows) swaps float4s
+      // so that lane i of the group writes the i-th 16 bytes of each of the four rows in turn: a
+      // store instruction covers 64 contiguous bytes of eight rows, not 16 bytes of 32 rows.
+      const int gi = lane & 3;
+      int64_t orow[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) orow[q] = __shfl_sync(0xFFFFFFFFu, out_row, (lane & ~3) | q);
 #pragma unroll
       for (int u = 0; u < D / 16; ++u) {
         if (u % NS != hs) continue;
         float o[16];
         tmem_ld16(o_t + 16 * u, o);
         tmem_wait_ld();
-        if (valid) {
-          float4* dst = reinterpret_cast<float4*>(a.out + out_row + 16 * u);
-          if (cl_q) {
-            // Sec. 3.1: a <CL> attends only to itself, so its output is its own value row
-            const uint4* vsrc = reinterpret_cast<const uint4*>(a.v + (w.row_base + iq) * D + 16 * u);
+        float4 f[4];
 #pragma unroll
-            for (int e2 = 0; e2 < 2; ++e2) {
-              const uint4 vv = __ldg(vsrc + e2);
-              const float2 f0 = T::f2(vv.x), f1 = T::f2(vv.y), f2 = T::f2(vv.z), f3 = T::f2(vv.w);
-              dst[2 * e2] = make_float4(f0.x, f0.y, f1.x, f1.y);
-              dst[2 * e2 + 1] = make_float4(f2.x, f2.y, f3.x, f3.y);
-            }
-          } else {
+        for (int e = 0; e < 4; ++e) f[e] = make_float4(o[4 * e] * inv, o[4 * e + 1] * inv, o[4 * e + 2] * inv, o[4 * e + 3] * inv);
+        // 4 x 4 transpose of float4s across the group: exchange with lane gi ^ m the float4s whose
+        // index differs from gi in bit m, for m = 2 then 1
 #pragma unroll
-            for (int e = 0; e < 4; ++e)
-              dst[e] = make_float4(o[4 * e] * inv, o[4 * e + 1] * inv, o[4 * e + 2] * inv, o[4 * e + 3] * inv);
+        for (int m = 2; m >= 1; m >>= 1) {
+          const bool hi = (gi & m) != 0;
+#pragma unroll
+          for (int j0 = 0; j0 < 4; ++j0) {
+            if (j0 & m) continue;
+            const int j1 = j0 | m;
+            const float4 snd = hi ? f[j0] : f[j1];
+            float4 rcv;
+            rcv.x = __shfl_xor_sync(0xFFFFFFFFu, snd.x, m);
+            rcv.y = __shfl_xor_sync(0xFFFFFFFFu, snd.y, m);
+            rcv.z = __shfl_xor_sync(0xFFFFFFFFu, snd.z, m);
+            rcv.w = __shfl_xor_sync(0xFFFFFFFFu, snd.w, m);
+            if (hi)
+              f[j0] = rcv;
+            else
+              f[j1] = rcv;
           }
         }
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (orow[q] >= 0) reinterpret_cast<float4*>(a.out + orow[q] + 16 * u)[gi] = f[q];
       }
       tc_fence_before();
       // the row sums are read before the next item's first maximum exchange reuses the buffer

@@ -135,3 +135,37 @@ def test_prefill_query_subsets_and_errors():
         kvc.kvc_prefill_attention(loc.handle, 0, q[:3 * H * d], [1, 1, 1], 0.125, out)
     assert e.value.status == 2
     assert run.cache.device_status() == 0
+
+
+@pytest.mark.parametrize("policy", [orc.POLICY_PAPER, orc.POLICY_KEEP_CL])
+def test_prefill_query_tile_offsets(policy):
+    """The first query row at several offsets within a 128-row key tile (1, 127, 129, 200): key tiles
+    that end exactly at the first query, query tiles straddling two key tiles, and <CL> queries (tokens
+    64k + 7) in each of them, which must see their own key alone."""
+    w = wl.opt13b(b=4, L=330, M=1)
+    run = harness.Runner(w, 0, policy)
+    run.load_prompt(compress=False)
+    H, d, L = w.H, w.d, 330
+    q0 = np.array([1, 127, 129, 200])
+    n_q = (L - q0).astype(np.int32)
+    tok_t = torch.tensor(np.concatenate([np.arange(a, L) for a in q0]), dtype=torch.int32, device="cuda")
+    tok_s = torch.tensor(np.repeat(np.arange(4), n_q), dtype=torch.int32, device="cuda")
+    q = torch.empty(int(n_q.sum()) * H * d, dtype=torch.float16, device="cuda")
+    synth.fill_tokens_cuda(w.seed, w.dtype, synth.scale_for(w.q_sigma), synth.tag(synth.Q_TENSOR, 0), tok_t, tok_s,
+                           H, d, q)
+    out = torch.full((int(n_q.sum()), H, d), float("nan"), dtype=torch.float32, device="cuda")
+    kvc.kvc_prefill_attention(run.cache.handle, 0, q, n_q, w.scale, out)
+    heads = [0, 13, 31]
+    got = out.cpu().numpy()[:, heads]
+    ref = ow.expected_prefill(w, 0, range(4), np.full(4, L), n_q, heads, policy)
+    _compare(got, ref, "f16", f"query tiles at {q0.tolist()}")
+    assert run.cache.device_status() == 0
+
+
+def test_prefill_blocks_of_512_cl_key_in_last_column():
+    """Blocks of 512 tokens: once the first block's spans are freed, the second block's queries start
+    at stored row 248, so the <CL> at token 519 is stored row 255, the last column of key tile 1.
+    Its query tile runs its key tiles in reverse, so the tile before holds no visible key for that
+    query and its own tile holds one, in the last column: the row maximum must take that column."""
+    w = wl.opt13b(b=2, L=1100, M=1)
+    run_prefill(w, 512, layers=[0], heads=[0, 31])
