@@ -33,9 +33,10 @@ namespace kvc {
 namespace {
 
 constexpr int kPfRows = 128;  // queries per tile (MMA M) and keys per tile (QK^T N, PV K)
-// Threads: a producer warp, an MMA warp, and NS softmax warpgroups that split each S row's 128
-// columns (NS threads per query row, one in each warpgroup).
-__host__ __device__ constexpr int pf_threads(int NS) { return 64 + 128 * NS; }
+// Threads: NS softmax warpgroups that split each S row's 128 columns (NS threads per query row,
+// one in each warpgroup), then one warpgroup holding the producer warp, the MMA warp and two idle
+// warps (so that registers can be moved between the two kinds of warpgroup).
+__host__ __device__ constexpr int pf_threads(int NS) { return 128 * NS + 128; }
 constexpr int kPfSplit = 1;
 
 // Shared-memory geometry for head dimension D.  Q, K and V tiles are [128 rows][D] split into
@@ -78,6 +79,15 @@ struct PfCfg {
   static_assert(TMEM_END <= TMEM_COLS && TMEM_COLS * CPS <= 512, "TMEM budget");
   static_assert(D % 16 == 0 && SW * NSUB == 2 * D, "bad tile geometry");
   static_assert(SMEM <= 227 * 1024 && (CPS == 1 || SMEM + 4096 <= 113 * 1024), "shared memory budget");
+  // Registers with two CTAs per SM: each thread is launched with REG_LAUNCH, then the producer's
+  // warpgroup gives registers up (setmaxnreg.dec to REG_OTHER) and the softmax warpgroup takes them
+  // (setmaxnreg.inc to REG_SOFTMAX); the two shares add up to exactly what the CTA was launched with.
+  static constexpr int REG_LAUNCH = 65536 / (CPS * pf_threads(kPfSplit));
+  static constexpr int REG_OTHER = 40;
+  static constexpr int REG_SOFTMAX = (REG_LAUNCH * pf_threads(kPfSplit) - REG_OTHER * 128) / (128 * kPfSplit) / 8 * 8;
+  static_assert(CPS == 1 || REG_SOFTMAX * 128 * kPfSplit + REG_OTHER * 128 <= REG_LAUNCH * pf_threads(kPfSplit),
+                "setmaxnreg shares exceed the launch allocation");
+  static_assert(CPS == 1 || (REG_SOFTMAX <= 256 && REG_SOFTMAX % 8 == 0 && REG_OTHER % 8 == 0), "setmaxnreg range");
 };
 
 // ---------------------------------------------------------------------------------------------
@@ -341,8 +351,14 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_slot;
+  // At the two-CTA register cap, registers go from the producer's warpgroup to the softmax: each
+  // role starts with its setmaxnreg (every warp of a warpgroup executes the same one).
+  auto regs_other = [] {
+    if constexpr (Cf::CPS == 2) asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(Cf::REG_OTHER));
+  };
 
-  if (warp == 0) {
+  if (warp == 4 * NS) {
+    regs_other();
     // ---------------- producer ----------------
     int64_t g = 0;  // tiles issued
     bool ok = true;
@@ -432,7 +448,8 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       for (int64_t t = g > NST ? g - NST : 0; t < g; ++t)
         mbar_wait_bounded(&full_bar[t % NST], (uint32_t)(t / NST) & 1, 100000000ull);
     }
-  } else if (warp == 1) {
+  } else if (warp == 4 * NS + 1) {
+    regs_other();
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       constexpr uint32_t idS = mma_idesc(Pack16<T>::kType, 0, kPfRows, kPfRows);
@@ -503,12 +520,13 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       tc_commit(&drain);
       mbar_wait_bounded(&drain, 0, a.wait_limit_ns);
     }
-  } else {
+  } else if (warp < 4 * NS) {
+    if constexpr (Cf::CPS == 2) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(Cf::REG_SOFTMAX));
     // ---------------- softmax: NS threads per query row ----------------
     constexpr int CW = kPfRows / NS;  // S columns of one thread
     constexpr int NSM = 128 * NS;     // softmax threads (named barrier 1)
     const int quarter = warp & 3;
-    const int hs = (warp - 2) >> 2;     // which column slice of the row
+    const int hs = warp >> 2;           // which column slice of the row
     const int r = quarter * 32 + lane;  // tile row == TMEM lane
     const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
     const float c2 = a.c2;
@@ -842,6 +860,8 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       w = wn;
       ++k;
     }
+  } else {
+    regs_other();  // the two idle warps of the producer's warpgroup
   }
   tc_fence_before();
   __syncthreads();
@@ -879,6 +899,14 @@ cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int6
     const cudaError_t e = cudaFuncSetAttribute(prefill_kernel<T, D, kPfSplit>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)PfCfg<D>::SMEM);
     if (e != cudaSuccess) return e;
+    if (PfCfg<D>::CPS == 2) {
+      // the setmaxnreg shares assume each thread starts with exactly REG_LAUNCH registers; with
+      // fewer the softmax warpgroup's increase could never be granted, so refuse to launch
+      cudaFuncAttributes fa;
+      const cudaError_t e2 = cudaFuncGetAttributes(&fa, prefill_kernel<T, D, kPfSplit>);
+      if (e2 != cudaSuccess) return e2;
+      if (fa.numRegs != PfCfg<D>::REG_LAUNCH) return cudaErrorInvalidConfiguration;
+    }
     attr_set = true;
   }
   CUtensorMap mk, mv;
