@@ -33,11 +33,9 @@ namespace kvc {
 namespace {
 
 constexpr int kPfRows = 128;  // queries per tile (MMA M) and keys per tile (QK^T N, PV K)
-// Threads: NS softmax warpgroups that split each S row's 128 columns (NS threads per query row,
-// one in each warpgroup), then one warpgroup holding the producer warp, the MMA warp and two idle
-// warps (so that registers can be moved between the two kinds of warpgroup).
-__host__ __device__ constexpr int pf_threads(int NS) { return 128 * NS + 128; }
-constexpr int kPfSplit = 1;
+// Threads: a softmax warpgroup (one thread per query row), then a warpgroup holding the producer
+// warp, the MMA warp and two idle warps (so that registers can be moved between the two).
+constexpr int kPfThreads = 256;
 
 // Shared-memory geometry for head dimension D.  Q, K and V tiles are [128 rows][D] split into
 // column subtiles of SW bytes per row, the widest swizzle (128 / 64 / 32 bytes) that divides a row;
@@ -82,10 +80,10 @@ struct PfCfg {
   // Registers with two CTAs per SM: each thread is launched with REG_LAUNCH, then the producer's
   // warpgroup gives registers up (setmaxnreg.dec to REG_OTHER) and the softmax warpgroup takes them
   // (setmaxnreg.inc to REG_SOFTMAX); the two shares add up to exactly what the CTA was launched with.
-  static constexpr int REG_LAUNCH = 65536 / (CPS * pf_threads(kPfSplit));
+  static constexpr int REG_LAUNCH = 65536 / (CPS * kPfThreads);
   static constexpr int REG_OTHER = 40;
-  static constexpr int REG_SOFTMAX = (REG_LAUNCH * pf_threads(kPfSplit) - REG_OTHER * 128) / (128 * kPfSplit) / 8 * 8;
-  static_assert(CPS == 1 || REG_SOFTMAX * 128 * kPfSplit + REG_OTHER * 128 <= REG_LAUNCH * pf_threads(kPfSplit),
+  static constexpr int REG_SOFTMAX = (REG_LAUNCH * kPfThreads - REG_OTHER * 128) / 128 / 8 * 8;
+  static_assert(CPS == 1 || REG_SOFTMAX * 128 + REG_OTHER * 128 <= REG_LAUNCH * kPfThreads,
                 "setmaxnreg shares exceed the launch allocation");
   static_assert(CPS == 1 || (REG_SOFTMAX <= 256 && REG_SOFTMAX % 8 == 0 && REG_OTHER % 8 == 0), "setmaxnreg range");
 };
@@ -298,8 +296,8 @@ __device__ __forceinline__ int pf_key_tile(int64_t it, int j, int nk) { return (
 // Persistent: each CTA walks its contiguous range of items (balanced by the host); every barrier
 // phase counts tiles over all of the CTA's items, so the producer streams the next item's K/V while
 // the current one finishes, and the O accumulator alternates between two TMEM buffers per item.
-template <typename T, int D, int NS>
-__global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
+template <typename T, int D>
+__global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
     prefill_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                    const PrefillArgs a) {
   using Cf = PfCfg<D>;
@@ -317,7 +315,6 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
   __shared__ uint32_t rcol[NST][kPfRows];
   __shared__ int32_t kn[NST];
   __shared__ int32_t kslow[NST];  // the tile needs the per-key rule (else its mask columns decide)
-  __shared__ float xbuf[NS > 1 ? 2 * NS * kPfRows : 1];
   __shared__ PfItem next_item;  // the item after the current one, as the softmax warps found it
   __shared__ int32_t qmeta[kPfRows];  // mask bounds of the query rows of the next item
   __shared__ uint32_t tmem_slot;
@@ -339,9 +336,9 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       mbar_init(&empty_bar[i], 1);
     }
     for (int i = 0; i < SBUF; ++i) mbar_init(&s_full[i], 1);
-    mbar_init(&s_free, 128 * NS);  // one S tile: the softmax has read it
-    mbar_init(&q_full, 128 * NS);
-    mbar_init(&p_full, 128 * NS);
+    mbar_init(&s_free, 128);  // one S tile: the softmax has read it
+    mbar_init(&q_full, 128);
+    mbar_init(&p_full, 128);
     mbar_init(&pv_done, 1);
     mbar_init(&drain, 1);
     abort_flag = 0;
@@ -357,7 +354,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
     if constexpr (Cf::CPS == 2) asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(Cf::REG_OTHER));
   };
 
-  if (warp == 4 * NS) {
+  if (warp == 4) {
     regs_other();
     // ---------------- producer ----------------
     int64_t g = 0;  // tiles issued
@@ -448,7 +445,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       for (int64_t t = g > NST ? g - NST : 0; t < g; ++t)
         mbar_wait_bounded(&full_bar[t % NST], (uint32_t)(t / NST) & 1, 100000000ull);
     }
-  } else if (warp == 4 * NS + 1) {
+  } else if (warp == 5) {
     regs_other();
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
@@ -520,19 +517,14 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       tc_commit(&drain);
       mbar_wait_bounded(&drain, 0, a.wait_limit_ns);
     }
-  } else if (warp < 4 * NS) {
+  } else if (warp < 4) {
     if constexpr (Cf::CPS == 2) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(Cf::REG_SOFTMAX));
-    // ---------------- softmax: NS threads per query row ----------------
-    constexpr int CW = kPfRows / NS;  // S columns of one thread
-    constexpr int NSM = 128 * NS;     // softmax threads (named barrier 1)
-    const int quarter = warp & 3;
-    const int hs = warp >> 2;           // which column slice of the row
-    const int r = quarter * 32 + lane;  // tile row == TMEM lane
-    const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
+    // ---------------- softmax: one thread per query row ----------------
+    constexpr int CW = kPfRows;  // S columns of one thread
+    constexpr int NSM = 128;     // softmax threads (named barrier 1)
+    const int r = warp * 32 + lane;  // tile row == TMEM lane
+    const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
     const float c2 = a.c2;
-    float* xmax = xbuf;  // [2][NS][128] row-maximum exchange; [NS][128] row sums at the end
-    // the query row of item w, rotated at its position (RoPE, pairs (e, e + rot/2)), rounded to the
-    // cache type, into the K-major tile; 8 columns at a time
     // The query rows of item w into the K-major Q tile (row r per thread), in two halves: q_issue
     // starts 16-byte asynchronous copies of the raw row into its swizzled slots (no registers, so
     // they can be issued early, while the previous item's last tile is still in the softmax);
@@ -547,53 +539,49 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       return smem_addr(sm + Cf::Q_OFF) + u * Cf::SUBB + r * SW + phys * 16;
     };
     auto q_issue = [&](const PfItem& w) {
-      if (hs == 0) {
-        const int iq = w.qr0 + r;
-        const bool valid = iq < w.qr_end;
-        const int64_t row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : 0;
+      const int iq = w.qr0 + r;
+      const bool valid = iq < w.qr_end;
+      const int64_t row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : 0;
 #pragma unroll
-        for (int c8 = 0; c8 < D / 8; ++c8) cp_async16(q_chunk(c8), a.q + row + 8 * c8, valid ? 16u : 0u);
-        cp_async4(smem_addr(&qmeta[r]), a.meta + (valid ? w.ps.moff + iq : 0), valid ? 4u : 0u);
-        cp_async_commit();
-      }
+      for (int c8 = 0; c8 < D / 8; ++c8) cp_async16(q_chunk(c8), a.q + row + 8 * c8, valid ? 16u : 0u);
+      cp_async4(smem_addr(&qmeta[r]), a.meta + (valid ? w.ps.moff + iq : 0), valid ? 4u : 0u);
+      cp_async_commit();
     };
     auto q_finish = [&](const PfItem& w) {
-      if (hs == 0) {
-        cp_async_wait_all();
-        const int half = a.rot / 2;
-        const int iq = w.qr0 + r;
-        if (half > 0 && iq < w.qr_end) {
-          const int32_t qpos = a.pos[a.off[w.s] + iq];
-          for (int c8 = 0; c8 < half / 8; ++c8) {
-            const uint32_t a1 = q_chunk(c8), a2 = q_chunk(c8 + half / 8);
-            const uint4 u1 = ld_shared_v4(a1), u2 = ld_shared_v4(a2);
-            const uint32_t w1[4] = {u1.x, u1.y, u1.z, u1.w}, w2[4] = {u2.x, u2.y, u2.z, u2.w};
-            uint32_t o1[4], o2[4];
+      cp_async_wait_all();
+      const int half = a.rot / 2;
+      const int iq = w.qr0 + r;
+      if (half > 0 && iq < w.qr_end) {
+        const int32_t qpos = a.pos[a.off[w.s] + iq];
+        for (int c8 = 0; c8 < half / 8; ++c8) {
+          const uint32_t a1 = q_chunk(c8), a2 = q_chunk(c8 + half / 8);
+          const uint4 u1 = ld_shared_v4(a1), u2 = ld_shared_v4(a2);
+          const uint32_t w1[4] = {u1.x, u1.y, u1.z, u1.w}, w2[4] = {u2.x, u2.y, u2.z, u2.w};
+          uint32_t o1[4], o2[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float2 x1 = T::f2(w1[e]), x2 = T::f2(w2[e]);
-              float sn0, cs0, sn1, cs1;
-              rope_sincos(qpos, a.rope_g[8 * c8 + 2 * e], &sn0, &cs0);
-              rope_sincos(qpos, a.rope_g[8 * c8 + 2 * e + 1], &sn1, &cs1);
-              o1[e] = Pack16<T>::two(x1.x * cs0 - x2.x * sn0, x1.y * cs1 - x2.y * sn1);
-              o2[e] = Pack16<T>::two(x2.x * cs0 + x1.x * sn0, x2.y * cs1 + x1.y * sn1);
-            }
-            st_shared_v4(a1, o1[0], o1[1], o1[2], o1[3]);
-            st_shared_v4(a2, o2[0], o2[1], o2[2], o2[3]);
+          for (int e = 0; e < 4; ++e) {
+            const float2 x1 = T::f2(w1[e]), x2 = T::f2(w2[e]);
+            float sn0, cs0, sn1, cs1;
+            rope_sincos(qpos, a.rope_g[8 * c8 + 2 * e], &sn0, &cs0);
+            rope_sincos(qpos, a.rope_g[8 * c8 + 2 * e + 1], &sn1, &cs1);
+            o1[e] = Pack16<T>::two(x1.x * cs0 - x2.x * sn0, x1.y * cs1 - x2.y * sn1);
+            o2[e] = Pack16<T>::two(x2.x * cs0 + x1.x * sn0, x2.y * cs1 + x1.y * sn1);
           }
+          st_shared_v4(a1, o1[0], o1[1], o1[2], o1[3]);
+          st_shared_v4(a2, o2[0], o2[1], o2[2], o2[3]);
         }
-        const uint32_t x01 = (uint32_t)T::r(256.f) | (qmeta[r] & 1 ? (uint32_t)T::r(256.f) << 16 : 0u);
-        if constexpr (Cf::XQT) {
-          const uint32_t wd[8] = {x01, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-          tmem_st8u(tl + Cf::XQ_COL, wd);
-          tmem_wait_st();
-          tc_fence_before();
-        } else {
-          const uint32_t row = smem_addr(sm + Cf::XQ_OFF) + r * 32;
-          const uint32_t sw = (r >> 2) & 1;  // 32-byte swizzle: the two 16-byte halves swap every 4 rows
-          st_shared_v4(row + 16 * sw, x01, 0u, 0u, 0u);
-          st_shared_v4(row + 16 * (sw ^ 1), 0u, 0u, 0u, 0u);
-        }
+      }
+      const uint32_t x01 = (uint32_t)T::r(256.f) | (qmeta[r] & 1 ? (uint32_t)T::r(256.f) << 16 : 0u);
+      if constexpr (Cf::XQT) {
+        const uint32_t wd[8] = {x01, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+        tmem_st8u(tl + Cf::XQ_COL, wd);
+        tmem_wait_st();
+        tc_fence_before();
+      } else {
+        const uint32_t row = smem_addr(sm + Cf::XQ_OFF) + r * 32;
+        const uint32_t sw = (r >> 2) & 1;  // 32-byte swizzle: the two 16-byte halves swap every 4 rows
+        st_shared_v4(row + 16 * sw, x01, 0u, 0u, 0u);
+        st_shared_v4(row + 16 * (sw ^ 1), 0u, 0u, 0u, 0u);
       }
       fence_proxy_async_smem();
       mbar_arrive(&q_full);
@@ -608,7 +596,6 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       w = pf_item(a, it);
       q_issue(w);
       q_finish(w);
-      if (NS > 1) bar_and(1, NSM, true);  // qmeta is read by every slice of the row
     }
     while (it < it1) {
       const bool has_next = it + 1 < it1;
@@ -629,7 +616,7 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
         if (wok) {
           tc_fence_after();
 #pragma unroll
-          for (int c = 0; c < CW; c += 32) tmem_ld32(tl + sb * kPfRows + hs * CW + c, sv + c);
+          for (int c = 0; c < CW; c += 32) tmem_ld32(tl + sb * kPfRows + c, sv + c);
           tmem_wait_ld();
           tc_fence_before();
         } else {
@@ -669,18 +656,12 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           v1 &= low_bits(t1 - 32) & ~low_bits(t0 - 32);
           v2 &= low_bits(t1 - 64) & ~low_bits(t0 - 64);
           v3 &= low_bits(t1 - 96) & ~low_bits(t0 - 96);
-          // this thread's words: columns [hs * CW, hs * CW + CW)
-          uint32_t vw[CW / 32];
-#pragma unroll
-          for (int q = 0; q < CW / 32; ++q) {
-            const int wd = hs * (CW / 32) + q;
-            vw[q] = wd == 0 ? v0 : wd == 1 ? v1 : wd == 2 ? v2 : v3;
-          }
+          const uint32_t vw[4] = {v0, v1, v2, v3};
 #pragma unroll
           for (int c = 0; c < CW; ++c) sv[c] = (vw[c >> 5] >> (c & 31)) & 1u ? sv[c] : -INFINITY;
         }
-        // row max: a tree over this slice (eight partial maxima: columns 0-7, then pairs of 8-column
-        // blocks, then the last block when one is left over), then across the NS slices of the row
+        // row max: a tree (eight partial maxima: columns 0-7, then pairs of 8-column blocks, then the
+        // last block when one is left over)
         static_assert(CW % 8 == 0, "slice width");
         constexpr int kPairEnd = 8 + (CW - 8) / 16 * 16;  // columns [8, kPairEnd) go in pairs of blocks
         float mx8[8];
@@ -694,24 +675,13 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
 #pragma unroll
           for (int u = 0; u < 8; ++u) mx8[u] = fmaxf(mx8[u], sv[kPairEnd + u]);
         }
-        float mx = max3(max3(mx8[0], mx8[1], mx8[2]), max3(mx8[3], mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]));
-        if (NS > 1) {
-          xmax[((gj & 1) * NS + hs) * kPfRows + r] = mx;
-          // every softmax thread passes this barrier: the exit decision is taken by all of them at once
-          if (!bar_and(1, NSM, ok)) {
-            ok = false;
-            break;
-          }
-        } else if (!__all_sync(0xFFFFFFFFu, ok)) {
-          // one slice per row: no exchange, so no barrier inside the tile loop -- a warp that stops
+        const float mx = max3(max3(mx8[0], mx8[1], mx8[2]), max3(mx8[3], mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]));
+        if (!__all_sync(0xFFFFFFFFu, ok)) {
+          // no exchange between the warps, so no barrier inside the tile loop -- a warp that stops
           // here meets the others at the barrier after the loop (their bounded waits give up at once
           // once any role has given up)
           ok = false;
           break;
-        }
-        if (NS > 1) {
-#pragma unroll
-          for (int q = 0; q < NS; ++q) mx = fmaxf(mx, xmax[((gj & 1) * NS + q) * kPfRows + r]);
         }
         // Reference maximum: moved only when the row maximum grows by more than 2^8 (log2 units), so
         // O is rescaled rarely; P stays below 2^8 and its scale cancels exactly in O / l.
@@ -734,7 +704,6 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
             tc_fence_after();
 #pragma unroll
             for (int u = 0; u < D / 16; ++u) {
-              if (u % NS != hs) continue;
               float o[16];
               tmem_ld16(o_t + 16 * u, o);
               tmem_wait_ld();
@@ -745,8 +714,8 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           }
         }
         // P = 2^(s c2 - ref) as 16-bit pairs (row r in lane r), stored 32 columns at a time as they
-        // are made; the row sum of this slice
-        const uint32_t p_tl = tl + (Cf::PSEP ? Cf::P_COL : sb * kPfRows) + hs * (CW / 2);
+        // are made; the row sum
+        const uint32_t p_tl = tl + (Cf::PSEP ? Cf::P_COL : sb * kPfRows);
         float2 rs4[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
         const float2 c2v = make_float2(c2, c2), nref = make_float2(-ref, -ref);
         const bool sok = __all_sync(0xFFFFFFFFu, ok);
@@ -764,17 +733,15 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           if (sok) tmem_st16u(p_tl + 16 * q, pk);
         }
         const float rs = ((rs4[0].x + rs4[0].y) + (rs4[1].x + rs4[1].y)) + ((rs4[2].x + rs4[2].y) + (rs4[3].x + rs4[3].y));
-        l = l * alpha + rs;  // this slice's part of the row sum
+        l = l * alpha + rs;
         tmem_wait_st();
         if (kb + kPfRows > w.ps.len && kb + r >= w.ps.len) {
           // a V row past the stored rows (stale or another stream's): zero it so 0 * V stays 0
           const uint32_t v_row = smem_addr(sm + Cf::KV_OFF + st * 2 * Cf::TILE + Cf::TILE) + r * SW;
 #pragma unroll
-          for (int u = 0; u < Cf::NSUB; ++u) {
-            if (u % NS != hs) continue;
+          for (int u = 0; u < Cf::NSUB; ++u)
 #pragma unroll
             for (int b16 = 0; b16 < SW / 16; ++b16) st_shared_v4(v_row + u * Cf::SUBB + b16 * 16, 0, 0, 0, 0);
-          }
           fence_proxy_async_smem();
         }
         if constexpr (SBUF == 2) {
@@ -796,21 +763,14 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       __syncwarp();
       const PfItem wn = has_next ? next_item : w;
       if (has_next) q_finish(wn);
-      // epilogue: O / l, with l summed over the NS slices of the row
+      // epilogue: O / l
       ok = pf_wait(&pv_done, (uint32_t)(g - 1) & 1, a, &abort_flag);
-      if (NS > 1) xmax[hs * kPfRows + r] = l;
       if (!bar_and(1, NSM, ok)) {
         ok = false;
         break;
       }
-      float lt = l;
-      if (NS > 1) {
-        lt = 0.f;
-#pragma unroll
-        for (int q = 0; q < NS; ++q) lt += xmax[q * kPfRows + r];
-      }
       tc_fence_after();
-      const float inv = 1.f / lt;
+      const float inv = 1.f / l;
       const int64_t out_row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : -1;
       // O / l to global memory.  Each group of four lanes (four consecutive query rows) swaps float4s
       // so that lane i of the group writes the i-th 16 bytes of each of the four rows in turn: a
@@ -821,7 +781,6 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
       for (int q = 0; q < 4; ++q) orow[q] = __shfl_sync(0xFFFFFFFFu, out_row, (lane & ~3) | q);
 #pragma unroll
       for (int u = 0; u < D / 16; ++u) {
-        if (u % NS != hs) continue;
         float o[16];
         tmem_ld16(o_t + 16 * u, o);
         tmem_wait_ld();
@@ -854,7 +813,8 @@ __global__ void __launch_bounds__(pf_threads(NS), PfCfg<D>::CPS)
           if (orow[q] >= 0) reinterpret_cast<float4*>(a.out + orow[q] + 16 * u)[gi] = f[q];
       }
       tc_fence_before();
-      // the row sums are read before the next item's first maximum exchange reuses the buffer
+      // every warp has read the next item (above) before any of them can overwrite it at the next
+      // item's last tile
       bar_and(1, NSM, true);
       it = next;
       w = wn;
@@ -896,14 +856,14 @@ template <typename T, int D>
 cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int64_t grid, cudaStream_t stream) {
   static bool attr_set = false;  // per instantiation; setting it twice is harmless
   if (!attr_set) {
-    const cudaError_t e = cudaFuncSetAttribute(prefill_kernel<T, D, kPfSplit>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    const cudaError_t e = cudaFuncSetAttribute(prefill_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)PfCfg<D>::SMEM);
     if (e != cudaSuccess) return e;
     if (PfCfg<D>::CPS == 2) {
       // the setmaxnreg shares assume each thread starts with exactly REG_LAUNCH registers; with
       // fewer the softmax warpgroup's increase could never be granted, so refuse to launch
       cudaFuncAttributes fa;
-      const cudaError_t e2 = cudaFuncGetAttributes(&fa, prefill_kernel<T, D, kPfSplit>);
+      const cudaError_t e2 = cudaFuncGetAttributes(&fa, prefill_kernel<T, D>);
       if (e2 != cudaSuccess) return e2;
       if (fa.numRegs != PfCfg<D>::REG_LAUNCH) return cudaErrorInvalidConfiguration;
     }
@@ -912,7 +872,7 @@ cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int6
   CUtensorMap mk, mv;
   std::memcpy(&mk, maps.k, sizeof mk);
   std::memcpy(&mv, maps.v, sizeof mv);
-  prefill_kernel<T, D, kPfSplit><<<(unsigned)grid, pf_threads(kPfSplit), PfCfg<D>::SMEM, stream>>>(mk, mv, a);
+  prefill_kernel<T, D><<<(unsigned)grid, kPfThreads, PfCfg<D>::SMEM, stream>>>(mk, mv, a);
   return cudaGetLastError();
 }
 
