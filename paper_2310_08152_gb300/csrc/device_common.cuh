@@ -31,16 +31,18 @@ struct BF16T {
 // ---------------------------------------------------------------------------------------------
 // RoPE angle.  theta = pos * base^(-2i/rot) is reduced in turns: g = base^(-2i/rot) / (2 pi) is
 // held as a double-float (hi, lo); pos * hi is split exactly with an FMA (Dekker's two-product),
-// the integer part of the turns is removed exactly, and sincospi takes the small remainder.  The
-// angle error stays near 1e-7 rad at any position below 2^24 (a plain binary32 product would be
-// off by up to half an ulp of theta, about 5e-4 rad at position 8192).
+// the integer part of the turns is removed exactly, leaving f in [-1/2, 1/2] turns with an error
+// near 1e-7 at any position below 2^24 (a plain binary32 product would be off by up to half an ulp
+// of theta, about 5e-4 rad at position 8192).  The sine and cosine of 2 pi f, an angle in
+// [-pi, pi], come from the hardware approximation, whose absolute error there (about 2^-21) is
+// far below the 16-bit rounding of the rotated values (2^-11 relative for fp16).
 // ---------------------------------------------------------------------------------------------
 __device__ __forceinline__ void rope_sincos(int32_t pos, float2 g, float* s, float* c) {
   const float p = (float)pos;
   const float a = __fmul_rn(p, g.x);
   const float e = __fmaf_rn(p, g.x, -a);
   const float f = __fadd_rn(__fsub_rn(a, rintf(a)), __fmaf_rn(p, g.y, e));
-  sincospif(2.0f * f, s, c);
+  __sincosf(6.28318530717958647692f * f, s, c);
 }
 
 // ---------------------------------------------------------------------------------------------
