@@ -30,75 +30,84 @@ namespace {
 
 constexpr unsigned kFull = 0xFFFFFFFFu;
 
+constexpr int kAppendThreads = 256;
+constexpr int64_t kAppendMaxBlocks = 16384;
+
 // ---------------------------------------------------------------------------------------------
 // a1: append
 // ---------------------------------------------------------------------------------------------
-// Work items: [0, n_copy) copy one 16-byte vector (all of V, the unrotated columns of K);
-// [n_copy, n_copy + n_rot) rotate one pair of 8-column vectors of K for every head of one token.
+// One (layer, token) unit per block iteration: its plan entry and row addresses are found once, then
+// the block's threads split the unit's 16-byte vectors -- every V vector and every unrotated K
+// vector of every head (copies), and every pair of rotated K vectors (vec, vec + rot/16) of every
+// head -- with 32-bit index arithmetic.  The token's RoPE sines and cosines (rot/2 of them) are
+// computed once per unit into shared memory.
 template <typename T, int D>
-__global__ void __launch_bounds__(256) append_kernel(Geometry g, Static st, Buffers buf,
-                                                     const TokPlan* __restrict__ plan, int64_t ntok, int64_t n_in,
-                                                     int m0, int n_layers, int write_meta,
-                                                     const uint16_t* __restrict__ k_in,
-                                                     const uint16_t* __restrict__ v_in) {
+__global__ void __launch_bounds__(kAppendThreads) append_kernel(Geometry g, Static st, Buffers buf,
+                                                                const TokPlan* __restrict__ plan, int64_t ntok,
+                                                                int64_t n_in, int m0, int n_layers, int write_meta,
+                                                                const uint16_t* __restrict__ k_in,
+                                                                const uint16_t* __restrict__ v_in) {
   constexpr int VPR = D / 8;
+  __shared__ float2 rope_cs[D / 2];  // (cos, sin) of the token's rotated pairs
   const int H = g.H;
-  const int hv = g.rot / 16;              // vectors per rotated half
-  const int kcopy = VPR - 2 * hv;         // unrotated K vectors per row
-  const int per_row = VPR + kcopy;        // copy items per (layer, token, head)
-  const int64_t n_copy = (int64_t)n_layers * ntok * H * per_row;
-  const int64_t n_rot = (int64_t)n_layers * ntok * hv;
+  const int hv = g.rot / 16;           // vectors per rotated half
+  const int kcopy = VPR - 2 * hv;      // unrotated K vectors per row
+  const int per_row = VPR + kcopy;     // copy items per head
+  const int n_copy = H * per_row;      // copy items per unit
+  const int n_items = n_copy + H * hv; // + rotation items per unit
   const int64_t plane = (int64_t)H * g.C;  // rows per (layer, K/V) plane
-  for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < n_copy + n_rot;
-       idx += (int64_t)gridDim.x * blockDim.x) {
-    if (idx < n_copy) {
-      const int c = (int)(idx % per_row);
-      int64_t r = idx / per_row;
-      const int h = (int)(r % H);
-      r /= H;
-      const int64_t tok = r % ntok;
-      const int l = (int)(r / ntok);
-      const TokPlan tp = plan[tok];
+  const int64_t n_units = (int64_t)n_layers * ntok;
+  for (int64_t u = blockIdx.x; u < n_units; u += gridDim.x) {
+    const int l = (int)(u / ntok);
+    const TokPlan tp = plan[u - (int64_t)l * ntok];
+    const uint16_t* k_src = k_in + ((int64_t)l * n_in + tp.in_tok) * H * D;  // head 0 of the token
+    const uint16_t* v_src = v_in + ((int64_t)l * n_in + tp.in_tok) * H * D;
+    const int64_t row0 = (int64_t)(m0 + l) * plane + st.seq_row0[tp.s] + tp.row;  // head 0's row
+    const int64_t hstride = st.cap[tp.s];                                        // rows between heads
+    if (hv > 0) {
+      __syncthreads();  // the previous unit's rotations are done with the table
+      for (int i = threadIdx.x; i < 8 * hv; i += blockDim.x) {
+        float sn, cs;
+        rope_sincos(tp.pos, st.rope_g[i], &sn, &cs);
+        rope_cs[i] = make_float2(cs, sn);
+      }
+      __syncthreads();
+    }
+    // copies: every V vector and every unrotated K vector of every head
+    for (int j = threadIdx.x; j < n_copy; j += blockDim.x) {
+      const int h = j / per_row, c = j - h * per_row;
       const bool is_v = c < VPR;
       const int vec = is_v ? c : 2 * hv + (c - VPR);
-      const uint16_t* src = (is_v ? v_in : k_in) + (((int64_t)l * n_in + tp.in_tok) * H + h) * D;
-      uint16_t* dst = (is_v ? buf.v : buf.k) +
-                      ((int64_t)(m0 + l) * plane + st.seq_row0[tp.s] + (int64_t)h * st.cap[tp.s] + tp.row) * D;
-      *reinterpret_cast<uint4*>(dst + vec * 8) = __ldg(reinterpret_cast<const uint4*>(src + vec * 8));
-      if (write_meta && l == 0 && h == 0 && c == 0) {
-        buf.pos[st.off[tp.s] + tp.row] = tp.pos;
-        buf.orig[st.off[tp.s] + tp.row] = tp.orig;
-      }
-    } else {
-      const int64_t w = idx - n_copy;
-      const int vec = (int)(w % hv);
-      const int64_t r = w / hv;
-      const int64_t tok = r % ntok;
-      const int l = (int)(r / ntok);
-      const TokPlan tp = plan[tok];
-      float cs[8], sn[8];
+      const uint16_t* src = (is_v ? v_src : k_src) + h * D + vec * 8;
+      uint16_t* dst = (is_v ? buf.v : buf.k) + (row0 + h * hstride) * D + vec * 8;
+      *reinterpret_cast<uint4*>(dst) = __ldg(reinterpret_cast<const uint4*>(src));
+    }
+    // rotations: one pair of vectors of one head per item
+    for (int j = n_copy + threadIdx.x; j < n_items; j += blockDim.x) {
+      const int jr = j - n_copy;
+      const int h = jr / hv, vec = jr - h * hv;
+      const uint16_t* src = k_src + h * D;
+      uint16_t* dst = buf.k + (row0 + h * hstride) * D;
+      const uint4 a = __ldg(reinterpret_cast<const uint4*>(src + vec * 8));
+      const uint4 b = __ldg(reinterpret_cast<const uint4*>(src + (vec + hv) * 8));
+      const uint16_t* xa = reinterpret_cast<const uint16_t*>(&a);
+      const uint16_t* xb = reinterpret_cast<const uint16_t*>(&b);
+      uint4 ya, yb;
+      uint16_t* pa = reinterpret_cast<uint16_t*>(&ya);
+      uint16_t* pb = reinterpret_cast<uint16_t*>(&yb);
 #pragma unroll
-      for (int e = 0; e < 8; ++e) rope_sincos(tp.pos, st.rope_g[vec * 8 + e], &sn[e], &cs[e]);
-      for (int h = 0; h < H; ++h) {
-        const uint16_t* src = k_in + (((int64_t)l * n_in + tp.in_tok) * H + h) * D;
-        uint16_t* dst =
-            buf.k + ((int64_t)(m0 + l) * plane + st.seq_row0[tp.s] + (int64_t)h * st.cap[tp.s] + tp.row) * D;
-        uint4 a = __ldg(reinterpret_cast<const uint4*>(src + vec * 8));
-        uint4 b = __ldg(reinterpret_cast<const uint4*>(src + (vec + hv) * 8));
-        const uint16_t* xa = reinterpret_cast<const uint16_t*>(&a);
-        const uint16_t* xb = reinterpret_cast<const uint16_t*>(&b);
-        uint4 ya, yb;
-        uint16_t* pa = reinterpret_cast<uint16_t*>(&ya);
-        uint16_t* pb = reinterpret_cast<uint16_t*>(&yb);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float x1 = T::f1(xa[e]), x2 = T::f1(xb[e]);
-          pa[e] = T::r(x1 * cs[e] - x2 * sn[e]);
-          pb[e] = T::r(x2 * cs[e] + x1 * sn[e]);
-        }
-        *reinterpret_cast<uint4*>(dst + vec * 8) = ya;
-        *reinterpret_cast<uint4*>(dst + (vec + hv) * 8) = yb;
+      for (int e = 0; e < 8; ++e) {
+        const float2 r = rope_cs[vec * 8 + e];
+        const float x1 = T::f1(xa[e]), x2 = T::f1(xb[e]);
+        pa[e] = T::r(x1 * r.x - x2 * r.y);
+        pb[e] = T::r(x2 * r.x + x1 * r.y);
       }
+      *reinterpret_cast<uint4*>(dst + vec * 8) = ya;
+      *reinterpret_cast<uint4*>(dst + (vec + hv) * 8) = yb;
+    }
+    if (write_meta && l == 0 && threadIdx.x == 0) {
+      buf.pos[st.off[tp.s] + tp.row] = tp.pos;
+      buf.orig[st.off[tp.s] + tp.row] = tp.orig;
     }
   }
 }
@@ -831,14 +840,11 @@ template <typename T, int D>
 cudaError_t launch_append_t(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t ntok,
                             int64_t n_in, int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
                             cudaStream_t stream) {
-  constexpr int VPR = D / 8;
-  const int hv = g.rot / 16;
-  const int64_t n_items =
-      (int64_t)n_layers * ntok * ((int64_t)g.H * (VPR + VPR - 2 * hv) + hv);
-  int64_t blocks = (n_items + 255) / 256;
-  if (blocks > 65535LL * 16) blocks = 65535LL * 16;
+  // one (layer, token) unit per block at a time; enough blocks for every SM several times over
+  int64_t blocks = (int64_t)n_layers * ntok;
+  if (blocks > kAppendMaxBlocks) blocks = kAppendMaxBlocks;
   if (blocks < 1) blocks = 1;
-  append_kernel<T, D><<<(unsigned)blocks, 256, 0, stream>>>(g, st, buf, plan, ntok, n_in, m0, n_layers, write_meta ? 1 : 0,
+  append_kernel<T, D><<<(unsigned)blocks, kAppendThreads, 0, stream>>>(g, st, buf, plan, ntok, n_in, m0, n_layers, write_meta ? 1 : 0,
                                                             static_cast<const uint16_t*>(k_in),
                                                             static_cast<const uint16_t*>(v_in));
   return cudaGetLastError();
