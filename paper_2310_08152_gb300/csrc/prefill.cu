@@ -1,17 +1,19 @@
 // sm_103a masked prefill attention on the 5th-generation tensor cores (Sec. 3.1: the modified
 // causal mask over every token of a prompt block).
 //
-// One CTA per (128-query tile, head, sequence).  The queries are the last tokens of each
-// sequence's history; the keys are the sequence's stored rows of one layer, read straight from the
-// ragged cache.  Per CTA:
+// Work items are (sequence, head, 128-query tile); the queries are the last tokens of each
+// sequence's history, the keys the sequence's stored rows of one layer, read straight from the
+// ragged cache.  Persistent CTAs (two per SM for d_head 64 and 80, one otherwise) each walk a
+// contiguous range of items that the host balances.  Per CTA:
 //
-//   warp 0       TMA producer: 2-D tiled copies (cp.async.bulk.tensor, swizzled) of 128-row K and V
-//                tiles into a ring of shared-memory stages, plus the tile's per-key mask bounds
-//   warp 1       one thread issues tcgen05.mma: S = Q K^T into a double-buffered TMEM tile, then
-//                O += P V into a TMEM accumulator; completions are signalled with tcgen05.commit
-//   warps 2..5   one query row per thread: tcgen05.ld of its S row, the sentinel mask, an online
-//                softmax in the exp2 domain, the rescale of its O row in TMEM, P (16-bit) into a
-//                swizzled shared-memory tile, and the final O / l
+//   warps 0..3   softmax, one query row per thread: tcgen05.ld of its S row, the per-key rule on the
+//                tiles that need it, an online softmax in the exp2 domain, P (16-bit) back into TMEM,
+//                the rare rescale of its O row, and the final O / l
+//   warp 4       TMA producer: 2-D tiled copies (cp.async.bulk.tensor, swizzled) of 128-row K and V
+//                tiles into a ring of shared-memory stages, the tile's mask columns and key classes
+//   warp 5       one thread issues tcgen05.mma: S = Q K^T (plus the mask columns) into TMEM, then
+//                O += P V with P read from TMEM; completions are signalled with tcgen05.commit
+//   warps 6, 7   idle (they complete the producer's warpgroup, whose registers go to the softmax)
 //
 // Mask (Sec. 3.1, the same rows a decode at the query would see): stored row i is visible to the
 // query at stored row iq exactly when i <= iq <= hid(i), except that a <CL> query sees only itself.
@@ -295,7 +297,8 @@ __device__ __forceinline__ int pf_key_tile(int64_t it, int j, int nk) { return (
 
 // Persistent: each CTA walks its contiguous range of items (balanced by the host); every barrier
 // phase counts tiles over all of the CTA's items, so the producer streams the next item's K/V while
-// the current one finishes, and the O accumulator alternates between two TMEM buffers per item.
+// the current one finishes (with two S tiles, the O accumulator also alternates between two TMEM
+// buffers per item).
 template <typename T, int D>
 __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
     prefill_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
