@@ -117,7 +117,7 @@ struct PrefillArgs {
   int64_t C;
   const PfItemRec* items;  // [n_items], sequence-major, then head, then the query tile with the most keys first
   int64_t n_items;         // (query tile, head) work items
-  const int32_t* cta_items; // [n_ctas + 1]: CTA c takes items [cta_items[c], cta_items[c+1])
+  unsigned long long* item_counter;  // zero at launch: the CTAs take items [0, n_items) in order from it
   int n_ctas;              // persistent grid size
   const int32_t* meta;     // per stored row: (hid << 1) | is_cl
   const uint16_t* q;       // [sum n_q][H][D]

@@ -58,9 +58,9 @@ struct WsLayout {
   size_t src_map = 0;    // int32 [C]: source row of each destination row of a compaction
   size_t counters = 0;   // int32 [b*H]
   size_t partials = 0;   // float [(kMaxDecodeWorkers + b*H) * (D + 4)]
-  size_t pre = 0;        // prefill plan: [int32 cta][PfItemRec items][int32 meta C]
-  size_t pre_cta = 0;    // offsets inside the plan; int32 [kMaxPrefillCtas + 1]: each CTA's item range
-  size_t pre_items = 0;  // PfItemRec [pre_max_items]
+  size_t pre_counter = 0;  // uint64: the prefill launch's next work item
+  size_t pre = 0;        // prefill plan: [PfItemRec items][int32 meta C]
+  size_t pre_items = 0;  // offsets inside the plan; PfItemRec [pre_max_items]
   int64_t pre_max_items = 0;
   size_t pre_meta = 0;
   size_t pre_bytes = 0;
@@ -91,11 +91,11 @@ WsLayout ws_layout(int b, int H, int D, int rot, int64_t C) {
   L.partials = take(4 * (size_t)(kvc::kMaxDecodeWorkers + (int64_t)b * H) * (size_t)(D + 4));
   // work items: H per query tile, and a sequence of capacity cap has at most ceil(cap / 128) query
   // tiles, so at most H * (C / 128 + b) in all
-  L.pre_cta = 0;
-  L.pre_items = align_up(4 * (size_t)(kvc::kMaxPrefillCtas + 1), 16);
+  L.pre_items = 0;
   L.pre_max_items = (int64_t)H * ((C + 127) / 128 + b);
   L.pre_meta = align_up(L.pre_items + sizeof(kvc::PfItemRec) * (size_t)L.pre_max_items, 16);
   L.pre_bytes = L.pre_meta + 4 * (size_t)C;
+  L.pre_counter = take(8);
   L.pre = take(L.pre_bytes);
   L.total = o;
   return L;
@@ -909,39 +909,21 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
       qtok += n_q[s];
       Pq[s + 1] = Pq[s] + (n_q[s] + 127) / 128;
     }
-    // Work items (sequence, head, query tile) in the kernel's order -- sequence, head, the tile with
-    // the most keys first -- split into contiguous ranges of equal work (key tiles + 1 per item),
-    // one per CTA of the persistent grid: balanced, and each CTA stays on a few (sequence, head)
-    // streams whose K/V rows it re-reads from L2.
+    // Work items (sequence, head, query tile) in the kernel's order: sequence, head, the tile with
+    // the most keys first.
     const int64_t n_items = (int64_t)H * Pq[b];
     if (n_items > c->ws.pre_max_items) return fail(KVC_ERR_INVALID_ARG, "prefill work items exceed the plan");
+    // a persistent grid: every SM's CTAs, which take the items in this order from the launch's
+    // counter, so the items in flight at any time are neighbours sharing K/V tiles in L2
     const int G = (int)std::min<int64_t>(
         std::min(c->num_sms * kvc::prefill_ctas_per_sm(c->cfg.d_head), kvc::kMaxPrefillCtas), n_items);
-    int32_t* cta = reinterpret_cast<int32_t*>(img + c->ws.pre_cta);
-    std::vector<int32_t> work_sq;  // per (s, query tile), heads alike
-    std::vector<int> sq_seq;
-    double W = 0.0;
-    for (int s = 0; s < b; ++s) {
-      const int nqt = Pq[s + 1] - Pq[s];
-      for (int qt = nqt - 1; qt >= 0; --qt) {
-        const int64_t q_end = std::min<int64_t>(ps[s].q0 + 128 * (int64_t)(qt + 1), ps[s].len);
-        work_sq.push_back((int32_t)((q_end + 127) / 128 + 1));
-        W += (double)H * work_sq.back();
-      }
-    }
-    cta[0] = 0;
     {
       kvc::PfItemRec* items = reinterpret_cast<kvc::PfItemRec*>(img + c->ws.pre_items);
-      int c_next = 1;
-      double acc = 0.0;
       int64_t item = 0;
-      size_t base = 0;
       for (int s = 0; s < b; ++s) {
         const int nqt = Pq[s + 1] - Pq[s];
         for (int h = 0; h < H; ++h)
           for (int k = 0; k < nqt; ++k, ++item) {
-            acc += work_sq[base + k];
-            while (c_next < G && acc >= W * c_next / G) cta[c_next++] = (int32_t)(item + 1);
             kvc::PfItemRec& r = items[item];
             const int qt = nqt - 1 - k;
             r.ps = ps[s];
@@ -955,9 +937,7 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
             r.row0_hi = (int32_t)((uint64_t)row0 >> 32);
             r.pad = 0;
           }
-        base += nqt;
       }
-      while (c_next <= G) cta[c_next++] = (int32_t)n_items;
     }
     c->pre_ctas = G;
     e = c->ring.commit(c->wsp(c->ws.pre), bytes, stream);
@@ -988,8 +968,10 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
   a.wait_limit_ns = 2000000000ull;
   (void)D;
   a.n_items = (int64_t)H * c->pre_tiles;
-  a.cta_items = reinterpret_cast<const int32_t*>(c->wsp(c->ws.pre + c->ws.pre_cta));
+  a.item_counter = reinterpret_cast<unsigned long long*>(c->wsp(c->ws.pre_counter));
   a.n_ctas = c->pre_ctas;
+  e = cudaMemsetAsync(a.item_counter, 0, sizeof(unsigned long long), stream);
+  if (e != cudaSuccess) return cuda_fail(e, "reset the prefill item counter");
   e = kvc::launch_prefill(c->geom(), c->maps, a, stream);
   if (e != cudaSuccess) return cuda_fail(e, "prefill kernel");
   c->launches += 1;

@@ -38,6 +38,9 @@ constexpr int kPfRows = 128;  // queries per tile (MMA M) and keys per tile (QK^
 // Threads: a softmax warpgroup (one thread per query row), then a warpgroup holding the producer
 // warp, the MMA warp and two idle warps (so that registers can be moved between the two).
 constexpr int kPfThreads = 256;
+// Work items reach the MMA and softmax warps through a ring of this many slots, filled by the
+// producer warp as it takes them from the launch's counter.
+constexpr int kItemRing = 4;
 
 // Shared-memory geometry for head dimension D.  Q, K and V tiles are [128 rows][D] split into
 // column subtiles of SW bytes per row, the widest swizzle (128 / 64 / 32 bytes) that divides a row;
@@ -295,10 +298,11 @@ __device__ __forceinline__ PfItem pf_item(const PrefillArgs& a, int64_t it) {
 // read last, while they are still in L2.
 __device__ __forceinline__ int pf_key_tile(int64_t it, int j, int nk) { return (it & 1) ? nk - 1 - j : j; }
 
-// Persistent: each CTA walks its contiguous range of items (balanced by the host); every barrier
-// phase counts tiles over all of the CTA's items, so the producer streams the next item's K/V while
-// the current one finishes (with two S tiles, the O accumulator also alternates between two TMEM
-// buffers per item).
+// Persistent: the CTAs take items in the table's order from the launch's counter, one at a time (the
+// producer warp takes an item when it starts streaming it and passes it on through the ring); every
+// barrier phase counts tiles over all of the CTA's items, so the producer streams the next item's
+// K/V while the current one finishes (with two S tiles, the O accumulator also alternates between
+// two TMEM buffers per item).
 template <typename T, int D>
 __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
     prefill_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
@@ -308,6 +312,10 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
   extern __shared__ uint8_t pf_smem_raw[];
   __shared__ uint64_t full_bar[NST], empty_bar[NST], s_full[SBUF], s_free;
   __shared__ uint64_t q_full, p_full, pv_done, drain;
+  // the CTA's k-th item in slot k % kItemRing (-1: none left); full: the producer has written it,
+  // empty: the MMA thread and the four softmax warps have read it
+  __shared__ int64_t item_ring[kItemRing];
+  __shared__ uint64_t item_full[kItemRing], item_empty[kItemRing];
   // Per stage, the tile's keys against its item's query tile [qr0, qr_end): khid has bit c set when
   // key c's bound holds for every query of the tile (hid >= qr_end - 1).  The keys whose bound falls
   // inside it (qr0 <= hid < qr_end - 1: a span closing among the queries) come in runs of one bound
@@ -325,7 +333,6 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
 
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(pf_smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t it0 = a.cta_items[blockIdx.x], it1 = a.cta_items[blockIdx.x + 1];  // this CTA's items
 
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_slot)),
@@ -344,6 +351,10 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
     mbar_init(&p_full, 128);
     mbar_init(&pv_done, 1);
     mbar_init(&drain, 1);
+    for (int i = 0; i < kItemRing; ++i) {
+      mbar_init(&item_full[i], 1);
+      mbar_init(&item_empty[i], 1 + 4);
+    }
     abort_flag = 0;
     fence_mbar_init();
   }
@@ -362,7 +373,22 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
     // ---------------- producer ----------------
     int64_t g = 0;  // tiles issued
     bool ok = true;
-    for (int64_t it = it0; ok && it < it1; ++it) {
+    for (uint32_t k = 0; ok; ++k) {
+      // take the next item and pass it on
+      const int slot = (int)(k % kItemRing);
+      if (k >= kItemRing && !pf_wait(&item_empty[slot], ((k / kItemRing) - 1) & 1, a, &abort_flag)) {
+        ok = false;
+        break;
+      }
+      int64_t it = -1;
+      if (lane == 0) {
+        const unsigned long long t = atomicAdd(a.item_counter, 1ull);
+        it = t < (unsigned long long)a.n_items ? (int64_t)t : -1;
+        item_ring[slot] = it;
+        mbar_arrive(&item_full[slot]);
+      }
+      it = __shfl_sync(0xFFFFFFFFu, it, 0);
+      if (it < 0) break;
       const PfItem w = pf_item(a, it);
       for (int j = 0; j < w.nk; ++j, ++g) {
         const int kt = pf_key_tile(it, j, w.nk);
@@ -457,9 +483,13 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
       const uint32_t q_s = smem_addr(sm + Cf::Q_OFF);
       const uint32_t xq_s = smem_addr(sm + Cf::XQ_OFF), xk_s = smem_addr(sm + Cf::XK_OFF);
       int64_t g = 0;
-      uint32_t k = 0;
       bool ok = true;
-      for (int64_t it = it0; ok && it < it1; ++it, ++k) {
+      for (uint32_t k = 0; ok; ++k) {
+        const int slot = (int)(k % kItemRing);
+        if (!(ok = pf_wait(&item_full[slot], (k / kItemRing) & 1, a, &abort_flag))) break;
+        const int64_t it = item_ring[slot];
+        mbar_arrive(&item_empty[slot]);
+        if (it < 0) break;
         const int nk = pf_item(a, it).nk;
         ok = pf_wait(&q_full, k & 1, a, &abort_flag);
         if (!ok) break;
@@ -590,18 +620,28 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
       mbar_arrive(&q_full);
     };
 
+    // the CTA's kk-th item from the ring (-1: none left, -2: the wait gave up); each softmax warp
+    // reads it once and releases the slot
+    auto take = [&](uint32_t kk) -> int64_t {
+      const int slot = (int)(kk % kItemRing);
+      if (!pf_wait(&item_full[slot], (kk / kItemRing) & 1, a, &abort_flag)) return -2;
+      const int64_t v = item_ring[slot];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&item_empty[slot]);
+      return v;
+    };
     bool ok = true;
     int64_t g = 0;  // tiles consumed
     uint32_t k = 0;  // items done
-    int64_t it = it0;
+    int64_t it = take(0);
     PfItem w{};
-    if (it < it1) {
+    if (it >= 0) {
       w = pf_item(a, it);
       q_issue(w);
       q_finish(w);
     }
-    while (it < it1) {
-      const bool has_next = it + 1 < it1;
+    while (it >= 0) {
+      int64_t it_next = -1;  // the next item, taken at this item's last tile
       const int iq = w.qr0 + r;  // stored row of this query
       const bool valid = iq < w.qr_end;
       const bool cl_q = valid && (qmeta[r] & 1);
@@ -628,11 +668,16 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
         }
         if (Cf::PSEP) mbar_arrive(&s_free);  // the next Q K^T may overwrite S
         // S of the item's last tile is in: every Q K^T of the item is complete, the next item's
-        // queries may go into the Q tile
-        if (has_next && j == w.nk - 1) {
-          const PfItem nx = pf_item(a, it + 1);
-          q_issue(nx);
-          if (lane == 0) next_item = nx;  // every warp writes the same item
+        // queries may go into the Q tile (the producer has taken that item by now: it takes the
+        // next one as soon as it has issued this item's last tile)
+        if (j == w.nk - 1) {
+          it_next = take(k + 1);
+          if (it_next == -2) ok = false;
+          if (it_next >= 0) {
+            const PfItem nx = pf_item(a, it_next);
+            q_issue(nx);
+            if (lane == 0) next_item = nx;  // every warp writes the same item
+          }
         }
         const int kb = kPfRows * pf_key_tile(it, j, w.nk);
         if (kslow[st]) {
@@ -762,7 +807,7 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
       g += w.nk;
       // the next item's queries go in as soon as this item's last S tile is read (every Q K^T of
       // this item is complete), so its first tiles overlap this item's epilogue
-      const int64_t next = it + 1;
+      const bool has_next = it_next >= 0;
       __syncwarp();
       const PfItem wn = has_next ? next_item : w;
       if (has_next) q_finish(wn);
@@ -819,7 +864,7 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
       // every warp has read the next item (above) before any of them can overwrite it at the next
       // item's last tile
       bar_and(1, NSM, true);
-      it = next;
+      it = it_next;
       w = wn;
       ++k;
     }
