@@ -909,8 +909,8 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
       qtok += n_q[s];
       Pq[s + 1] = Pq[s] + (n_q[s] + 127) / 128;
     }
-    // Work items (sequence, head, query tile) in the kernel's order: sequence, head, the tile with
-    // the most keys first.
+    // Work items (sequence, head, query tile) in the kernel's order: sequence (longest first), head,
+    // the tile with the most keys first.
     const int64_t n_items = (int64_t)H * Pq[b];
     if (n_items > c->ws.pre_max_items) return fail(KVC_ERR_INVALID_ARG, "prefill work items exceed the plan");
     // a persistent grid: every SM's CTAs, which take the items in this order from the launch's
@@ -918,9 +918,14 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
     const int G = (int)std::min<int64_t>(
         std::min(c->num_sms * kvc::prefill_ctas_per_sm(c->cfg.d_head), kvc::kMaxPrefillCtas), n_items);
     {
+      // sequences with the most stored rows first, so the heaviest items are taken early and the
+      // last ones taken are short
+      std::vector<int> order(b);
+      for (int s = 0; s < b; ++s) order[s] = s;
+      std::stable_sort(order.begin(), order.end(), [&](int x, int y) { return ps[x].len > ps[y].len; });
       kvc::PfItemRec* items = reinterpret_cast<kvc::PfItemRec*>(img + c->ws.pre_items);
       int64_t item = 0;
-      for (int s = 0; s < b; ++s) {
+      for (int s : order) {
         const int nqt = Pq[s + 1] - Pq[s];
         for (int h = 0; h < H; ++h)
           for (int k = 0; k < nqt; ++k, ++item) {
