@@ -516,7 +516,11 @@ def run_kvc(args, w):
     torch.cuda.synchronize()
     compaction["prompt_append_ms"] = sum(a.elapsed_time(b) for a, b in append_ev)
     prompt_free = time_prompt_write_time_freeing(w, steps_total, dev)
-    prefill = [time_prompt_prefill(w, steps_total, dev, blk) for blk in (0, 512)]
+    if w.extra.get("policy") == "local":
+        # the local-attention cache keeps a window, not the sentinel structure the prefill mask reads
+        prefill = "not defined for the local-attention cache"
+    else:
+        prefill = [time_prompt_prefill(w, steps_total, dev, blk) for blk in (0, 512)]
     inputs = [run.make_step_inputs(g) for g in range(steps_total)]
     out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device=dev)
     torch.cuda.synchronize()
