@@ -67,25 +67,28 @@ def test_full_ragged():
 # sequences and two heads against the oracle's single-query attention over the mask.
 # --------------------------------------------------------------------------
 
-@pytest.mark.parametrize("block", [0, 512])
-def test_full_prefill_opt13b_shaped(block):
+@pytest.mark.parametrize("name,block", [("opt1.3b", 0), ("opt1.3b", 512), ("rope3b_I32", 0), ("rope3b_I32", 512)])
+def test_full_prefill(name, block):
+    """d_head 64 (OPT-1.3B shape) and d_head 80 with RoPE (3B rotary shape, r = 0.5), in one go and in
+    blocks of 512 tokens; only the sampled sequences' outputs are read back."""
     import oracle as orc
 
-    w = wl.opt13b()
+    w = wl.by_name(name)
     layers, seqs, heads = {0, w.M // 2, w.M - 1}, [0, w.b // 2, w.b - 1], [0, w.H - 1]
     run = harness.Runner(w, 0)
     got = []
 
     def keep(start, n, m, out):
         if m in layers:
-            got.append((start.copy(), n.copy(), m, out.cpu().numpy()))
+            row0 = np.concatenate([[0], np.cumsum(n)[:-1]])
+            sel = {s: out[int(row0[s]):int(row0[s] + n[s])][:, heads].cpu().numpy() for s in seqs}
+            got.append((start.copy(), n.copy(), m, sel))
 
     run.prefill_prompt(block=block, out_cb=keep)
     assert run.cache.device_status() == 0
     rng = np.random.default_rng(block + 1)
     n_checked = 0
-    for start, n, m, o in got:
-        row0 = np.concatenate([[0], np.cumsum(n)[:-1]])
+    for start, n, m, sel in got:
         for s in seqs:
             T = int(start[s] + n[s])
             kinds = np.asarray(w.prompt_kinds[s][:T], np.uint8)
@@ -99,7 +102,6 @@ def test_full_prefill_opt13b_shaped(block):
                 q = ow.q_bits(w, m, s, t, heads)
                 ref = np.stack([orc.attend(q[i], K[i], V[i], pos, rows, w.dtype, w.scale, w.rotary_dim, w.rope_base,
                                            int(pos[t])) for i in range(len(heads))])
-                g = o[row0[s] + (t - lo)][heads]
-                compare(g, ref, f"prefill block={block} layer {m} seq {s} token {t}")
+                compare(sel[s][t - lo], ref, f"{name} prefill block={block} layer {m} seq {s} token {t}")
                 n_checked += 1
     assert n_checked > 100
