@@ -113,9 +113,9 @@ struct PfItemRec {
 static_assert(sizeof(PfItemRec) == 48, "three 16-byte loads");
 
 struct PrefillArgs {
-  int layer, H, b, rot;
+  int layer, H, rot;
   int64_t C;
-  const PfItemRec* items;  // [n_items], sequence-major, then head, then the query tile with the most keys first
+  const PfItemRec* items;  // [n_items]: sequences with the most stored rows first, then head, then the query tile with the most keys first
   int64_t n_items;         // (query tile, head) work items
   unsigned long long* item_counter;  // zero at launch: the CTAs take items [0, n_items) in order from it
   int n_ctas;              // persistent grid size
@@ -124,9 +124,7 @@ struct PrefillArgs {
   float* out;              // [sum n_q][H][D]
   float c2;                // scale * log2(e)
   const int32_t* pos;      // [C] stored-row positions
-  const int64_t* off;      // [b]
-  const int64_t* seq_row0; // [b]
-  const int32_t* cap;      // [b]
+  const int64_t* off;      // [b]: a sequence's first entry in pos
   const float2* rope_g;    // [rot/2]
   int* status;
   unsigned long long wait_limit_ns;

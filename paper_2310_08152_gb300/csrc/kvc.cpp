@@ -955,7 +955,6 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
   kvc::PrefillArgs a;
   a.layer = layer;
   a.H = H;
-  a.b = b;
   a.rot = c->cfg.rotary_dim;
   a.C = c->C;
   a.items = reinterpret_cast<const kvc::PfItemRec*>(c->wsp(c->ws.pre + c->ws.pre_items));
@@ -966,8 +965,6 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
   a.pos = c->cfg.pos_base;
   const kvc::Static sta = c->stat();
   a.off = sta.off;
-  a.seq_row0 = sta.seq_row0;
-  a.cap = sta.cap;
   a.rope_g = sta.rope_g;
   a.status = c->bufs().status;
   a.wait_limit_ns = 2000000000ull;
