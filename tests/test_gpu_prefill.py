@@ -1,7 +1,8 @@
 """Parity of the tensor-core masked prefill (kvc_prefill_attention, through the C ABI) with the fp64
 oracle: every query of a prompt block under the sentinel mask (Sec. 3.1), in one go and block by
 block with the spans each block closed freed in between, ragged lengths and query tiles that start
-mid-tile, RoPE, both policies, every built d_head and both 16-bit types."""
+mid-tile, RoPE (full and partial rotary dimension, f16 and bf16), both policies, every built d_head
+and both 16-bit types."""
 import dataclasses
 
 import numpy as np
@@ -169,3 +170,15 @@ def test_prefill_blocks_of_512_cl_key_in_last_column():
     query and its own tile holds one, in the last column: the row maximum must take that column."""
     w = wl.opt13b(b=2, L=1100, M=1)
     run_prefill(w, 512, layers=[0], heads=[0, 31])
+
+
+def test_prefill_rope_bf16():
+    # the query rotation rounded to bf16 (held to eight times the f16 bound)
+    w = dataclasses.replace(wl.rope3b(32, b=2, L=400, M=1), dtype="bf16", name="rope-bf16")
+    run_prefill(w, 0, layers=[0], heads=[0, 31])
+
+
+def test_prefill_rope_partial_rotary_dim():
+    # only the first 32 of 80 dimensions rotated (pairs (e, e + 16)); blocks of 200 tokens
+    w = dataclasses.replace(wl.rope3b(32, b=2, L=384, M=1), rotary_dim=32, name="rope-partial")
+    run_prefill(w, 200, layers=[0], heads=[5, 30])
