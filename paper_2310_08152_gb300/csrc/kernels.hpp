@@ -122,6 +122,7 @@ struct PrefillArgs {
   const int32_t* meta;     // per stored row: (hid << 1) | is_cl
   const uint16_t* q;       // [sum n_q][H][D]
   float* out;              // [sum n_q][H][D]
+  int64_t n_qtok;          // sum n_q
   float c2;                // scale * log2(e)
   const int32_t* pos;      // [C] stored-row positions
   const int64_t* off;      // [b]: a sequence's first entry in pos

@@ -961,6 +961,8 @@ kvc_status kvc_prefill_attention(kvc_cache* c, int layer, const void* q, const i
   a.meta = reinterpret_cast<const int32_t*>(c->wsp(c->ws.pre + c->ws.pre_meta));
   a.q = static_cast<const uint16_t*>(q);
   a.out = out;
+  a.n_qtok = 0;
+  for (int s = 0; s < b; ++s) a.n_qtok += n_q[s];
   a.c2 = (float)((double)scale * 1.4426950408889634);
   a.pos = c->cfg.pos_base;
   const kvc::Static sta = c->stat();

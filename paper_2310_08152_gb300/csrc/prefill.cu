@@ -66,7 +66,13 @@ struct PfCfg {
   // by the Q.K^T product itself.
   static constexpr uint32_t XQ_OFF = KV_OFF + NST * 2 * TILE;
   static constexpr uint32_t XK_OFF = XQ_OFF + (XQT ? 0 : kPfRows * 32);
-  static constexpr uint32_t SMEM = XK_OFF + NST * kPfRows * 32 + 1024;  // + slack to align the base to 1024
+  // d_head 64 has shared memory to spare for O / l: each softmax warp stages 32 rows x 32 columns
+  // (4 KB, 128-byte swizzle) for a TMA tensor store
+  static constexpr bool OSTAGE = D == 64;
+  static constexpr uint32_t OST_OFF = (XK_OFF + NST * kPfRows * 32 + 1023) / 1024 * 1024;
+  static constexpr uint32_t OST_WARP = 32 * 32 * 4;
+  static constexpr uint32_t SMEM = (OSTAGE ? OST_OFF + 4 * OST_WARP : XK_OFF + NST * kPfRows * 32) +
+                                   1024;  // + slack to align the base to 1024
   // TMEM.  d_head 64 (two CTAs per SM, 256 columns each): S [0,128), P [128,192) (16-bit, two
   // per column), O [192,256) -- S is released as soon as the softmax has read it, so the next
   // Q.K^T overlaps the softmax.  d_head 80 (two CTAs per SM): S [0,128) with P written over its
@@ -110,6 +116,16 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
       : "memory");
 }
+// Tensor store from shared memory (bulk group of the issuing thread) and its waits.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, uint32_t src, int x, int y, int z) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z), "r"(src)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_commit(uint64_t* bar) {
@@ -306,7 +322,7 @@ __device__ __forceinline__ int pf_key_tile(int64_t it, int j, int nk) { return (
 template <typename T, int D>
 __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
     prefill_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
-                   const PrefillArgs a) {
+                   const __grid_constant__ CUtensorMap tm_o, const PrefillArgs a) {
   using Cf = PfCfg<D>;
   constexpr int SW = Cf::SW, SUB = Cf::SUB, NST = Cf::NST, SBUF = Cf::SBUF;
   extern __shared__ uint8_t pf_smem_raw[];
@@ -819,46 +835,73 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
       }
       tc_fence_after();
       const float inv = 1.f / l;
-      const int64_t out_row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : -1;
-      // O / l to global memory.  Each group of four lanes (four consecutive query rows) swaps float4s
-      // so that lane i of the group writes the i-th 16 bytes of each of the four rows in turn: a
-      // store instruction covers 64 contiguous bytes of eight rows, not 16 bytes of 32 rows.
-      const int gi = lane & 3;
-      int64_t orow[4];
+      if (Cf::OSTAGE && w.qr_end - w.qr0 == kPfRows) {
+        // a full tile: 32 columns at a time, each warp's 32 rows through its swizzled staging buffer
+        // into one TMA tensor store of box (32 columns, head h, 32 tokens)
+        const uint32_t stage_buf = smem_addr(sm + Cf::OST_OFF + warp * Cf::OST_WARP);
+        const int tok = w.ps.qtok + (w.qr0 - w.ps.q0) + 32 * warp;  // token of the warp's first row
 #pragma unroll
-      for (int q = 0; q < 4; ++q) orow[q] = __shfl_sync(0xFFFFFFFFu, out_row, (lane & ~3) | q);
+        for (int hc = 0; hc < D / 32; ++hc) {
+          float o[32];
+          tmem_ld16(o_t + 32 * hc, o);
+          tmem_ld16(o_t + 32 * hc + 16, o + 16);
+          tmem_wait_ld();
+          if (lane == 0) bulk_wait_read0();  // the warp's previous store has read the buffer
+          __syncwarp();
 #pragma unroll
-      for (int u = 0; u < D / 16; ++u) {
-        float o[16];
-        tmem_ld16(o_t + 16 * u, o);
-        tmem_wait_ld();
-        float4 f[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) f[e] = make_float4(o[4 * e] * inv, o[4 * e + 1] * inv, o[4 * e + 2] * inv, o[4 * e + 3] * inv);
-        // 4 x 4 transpose of float4s across the group: exchange with lane gi ^ m the float4s whose
-        // index differs from gi in bit m, for m = 2 then 1
-#pragma unroll
-        for (int m = 2; m >= 1; m >>= 1) {
-          const bool hi = (gi & m) != 0;
-#pragma unroll
-          for (int j0 = 0; j0 < 4; ++j0) {
-            if (j0 & m) continue;
-            const int j1 = j0 | m;
-            const float4 snd = hi ? f[j0] : f[j1];
-            float4 rcv;
-            rcv.x = __shfl_xor_sync(0xFFFFFFFFu, snd.x, m);
-            rcv.y = __shfl_xor_sync(0xFFFFFFFFu, snd.y, m);
-            rcv.z = __shfl_xor_sync(0xFFFFFFFFu, snd.z, m);
-            rcv.w = __shfl_xor_sync(0xFFFFFFFFu, snd.w, m);
-            if (hi)
-              f[j0] = rcv;
-            else
-              f[j1] = rcv;
+          for (int k = 0; k < 8; ++k)
+            st_shared_v4(stage_buf + lane * 128 + ((k ^ (lane & 7)) << 4), __float_as_uint(o[4 * k] * inv),
+                         __float_as_uint(o[4 * k + 1] * inv), __float_as_uint(o[4 * k + 2] * inv),
+                         __float_as_uint(o[4 * k + 3] * inv));
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_3d(&tm_o, stage_buf, 32 * hc, w.h, tok);
+            bulk_commit();
           }
         }
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-          if (orow[q] >= 0) reinterpret_cast<float4*>(a.out + orow[q] + 16 * u)[gi] = f[q];
+      } else {
+        const int64_t out_row = valid ? ((int64_t)(w.ps.qtok + (iq - w.ps.q0)) * a.H + w.h) * D : -1;
+        // O / l to global memory.  Each group of four lanes (four consecutive query rows) swaps float4s
+        // so that lane i of the group writes the i-th 16 bytes of each of the four rows in turn: a
+        // store instruction covers 64 contiguous bytes of eight rows, not 16 bytes of 32 rows.
+        const int gi = lane & 3;
+        int64_t orow[4];
+  #pragma unroll
+        for (int q = 0; q < 4; ++q) orow[q] = __shfl_sync(0xFFFFFFFFu, out_row, (lane & ~3) | q);
+  #pragma unroll
+        for (int u = 0; u < D / 16; ++u) {
+          float o[16];
+          tmem_ld16(o_t + 16 * u, o);
+          tmem_wait_ld();
+          float4 f[4];
+  #pragma unroll
+          for (int e = 0; e < 4; ++e) f[e] = make_float4(o[4 * e] * inv, o[4 * e + 1] * inv, o[4 * e + 2] * inv, o[4 * e + 3] * inv);
+          // 4 x 4 transpose of float4s across the group: exchange with lane gi ^ m the float4s whose
+          // index differs from gi in bit m, for m = 2 then 1
+  #pragma unroll
+          for (int m = 2; m >= 1; m >>= 1) {
+            const bool hi = (gi & m) != 0;
+  #pragma unroll
+            for (int j0 = 0; j0 < 4; ++j0) {
+              if (j0 & m) continue;
+              const int j1 = j0 | m;
+              const float4 snd = hi ? f[j0] : f[j1];
+              float4 rcv;
+              rcv.x = __shfl_xor_sync(0xFFFFFFFFu, snd.x, m);
+              rcv.y = __shfl_xor_sync(0xFFFFFFFFu, snd.y, m);
+              rcv.z = __shfl_xor_sync(0xFFFFFFFFu, snd.z, m);
+              rcv.w = __shfl_xor_sync(0xFFFFFFFFu, snd.w, m);
+              if (hi)
+                f[j0] = rcv;
+              else
+                f[j1] = rcv;
+            }
+          }
+  #pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (orow[q] >= 0) reinterpret_cast<float4*>(a.out + orow[q] + 16 * u)[gi] = f[q];
+        }
       }
       tc_fence_before();
       // every warp has read the next item (above) before any of them can overwrite it at the next
@@ -868,6 +911,7 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
       w = wn;
       ++k;
     }
+    if (Cf::OSTAGE && lane == 0) bulk_wait0();  // this warp's tensor stores are complete
   } else {
     regs_other();  // the two idle warps of the producer's warpgroup
   }
@@ -917,10 +961,23 @@ cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int6
     }
     attr_set = true;
   }
-  CUtensorMap mk, mv;
+  CUtensorMap mk, mv, mo;
   std::memcpy(&mk, maps.k, sizeof mk);
   std::memcpy(&mv, maps.v, sizeof mv);
-  prefill_kernel<T, D><<<(unsigned)grid, kPfThreads, PfCfg<D>::SMEM, stream>>>(mk, mv, a);
+  std::memset(&mo, 0, sizeof mo);
+  if (PfCfg<D>::OSTAGE && a.n_qtok >= kPfRows) {
+    // out as [token][head][D] fp32, stored in boxes of 32 columns x one head x 32 tokens from the
+    // softmax warps' swizzled staging buffers (only full query tiles take this path)
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.H, (cuuint64_t)a.n_qtok};
+    cuuint64_t strides[2] = {(cuuint64_t)D * 4, (cuuint64_t)a.H * D * 4};
+    cuuint32_t box[3] = {32, 1, 32};
+    cuuint32_t elem[3] = {1, 1, 1};
+    const CUresult r = g_encode(&mo, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, a.out, dims, strides, box, elem,
+                                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  }
+  prefill_kernel<T, D><<<(unsigned)grid, kPfThreads, PfCfg<D>::SMEM, stream>>>(mk, mv, mo, a);
   return cudaGetLastError();
 }
 
