@@ -597,7 +597,7 @@ def run_kvc(args, w):
                          "traffic": recorded_traffic(w.name),
                          "bytes_per_launch_mean": dec_bytes_total / launches_decode,
                          "launch_us_mean": dec_total_s / launches_decode * 1e6},
-            "decode_plan": {"mode": ["stream-K", "warp per segment (wide)", "warp per segment (narrow)"][plan["mode"]]
+            "decode_plan": {"mode": ["stream-K", "warp per segment (wide)", "warp per segment (narrow)", "whole segments, several per warp"][plan["mode"]]
                             if plan["mode"] >= 0 else None, "warps": plan["workers"],
                             "tile_rows": plan["tile_rows"], "stages": plan["stages"]},
             "decode_share_of_step": dec_total_s / elapsed,

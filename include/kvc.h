@@ -291,8 +291,8 @@ int64_t kvc_launch_count(const kvc_cache* cache);
 /* How the last decode launch divided its work (host-side record, no synchronisation):
  * plan[0] = mode (0: the kept rows split evenly over a full wave of warps, split (sequence, head)
  * segments merged by a log-sum-exp combine; 1 / 2: one warp per segment with the wide / narrow
- * shared-memory pipeline; -1: nothing launched yet), plan[1] = warps, plan[2] = rows per tile,
- * plan[3] = pipeline stages per warp. */
+ * shared-memory pipeline; 3: several consecutive whole segments per warp, no combine; -1: nothing
+ * launched yet), plan[1] = warps, plan[2] = rows per tile, plan[3] = pipeline stages per warp. */
 kvc_status kvc_last_decode_plan(const kvc_cache* cache, int32_t* plan);
 
 #ifdef __cplusplus

@@ -333,7 +333,7 @@ struct DecodeDev {
   float qscale;  // scale * log2(e)
   unsigned long long limit_ns;
   int kv_before_wait;  // the K/V rows may be streamed before the preceding grid completes
-  int seg_per_worker;  // 1: worker w owns segment w whole; 0: stream-K split of the rows
+  int seg_per_worker;  // k > 0: worker w owns segments [w k, w k + k) whole; 0: stream-K split of the rows
 };
 
 // The tiles of a worker: its flat row range [x, hi) of the concatenation over (sequence, head)
@@ -387,11 +387,15 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   }
   const int H = g.H;
   int64_t lo, hi;
-  if (p.seg_per_worker) {  // segment wid = (s, h) whole
-    const int s0 = wid / H;
-    const int64_t a = p.P[s0], z = p.P[s0 + 1];
-    lo = (int64_t)H * a + (int64_t)(wid % H) * (z - a);
-    hi = lo + (z - a);
+  int s_first = 0;
+  if (p.seg_per_worker) {  // segments [sg0, sg1] = (s, h) pairs in order, each whole
+    const int64_t sg0 = (int64_t)wid * p.seg_per_worker;
+    const int64_t sg1 = min(sg0 + p.seg_per_worker, (int64_t)g.b * H) - 1;
+    s_first = (int)(sg0 / H);
+    const int s1 = (int)(sg1 / H);
+    const int64_t a0 = p.P[s_first], z0 = p.P[s_first + 1], a1 = p.P[s1], z1 = p.P[s1 + 1];
+    lo = (int64_t)H * a0 + (sg0 - (int64_t)s_first * H) * (z0 - a0);
+    hi = (int64_t)H * a1 + (sg1 - (int64_t)s1 * H + 1) * (z1 - a1);
   } else {
     lo = (int64_t)wid * p.R / p.NW;
     hi = (int64_t)(wid + 1) * p.R / p.NW;
@@ -419,7 +423,7 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   // segment holding row `lo`: s = (number of sequences with H*P[s] <= lo) - 1
   int cnt = 0;
   if (p.seg_per_worker) {
-    cnt = wid / H + 1;
+    cnt = s_first + 1;
   } else {
     for (int base_s = 0; base_s < g.b; base_s += 32) {
       const int k = base_s + lane;
@@ -764,7 +768,7 @@ cudaError_t decode_occupancy(int* occ_out) {
 
 template <typename T, int D, int KPT, int S>
 cudaError_t launch_decode_cfg(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a,
-                              int64_t NW, bool by_segment, cudaStream_t stream, int* grid) {
+                              int64_t NW, int seg_per_worker, cudaStream_t stream, int* grid) {
   using C = DecodeCfg<D, KPT, S>;
   DecodeDev p;
   const int64_t plane = (int64_t)g.H * g.C * D;
@@ -782,7 +786,7 @@ cudaError_t launch_decode_cfg(const Geometry& g, const Static& st, const Buffers
   p.qscale = a.scale * 1.4426950408889634f;
   p.limit_ns = a.wait_limit_ns;
   p.kv_before_wait = a.kv_before_wait;
-  p.seg_per_worker = by_segment ? 1 : 0;
+  p.seg_per_worker = seg_per_worker;
   const int64_t ctas = (NW + C::WARPS - 1) / C::WARPS;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)ctas);
@@ -798,32 +802,52 @@ cudaError_t launch_decode_cfg(const Geometry& g, const Static& st, const Buffers
   return cudaLaunchKernelEx(&cfg, decode_kernel<T, D, KPT, S>, g, st, p);
 }
 
+// k whole segments per worker, k as small as one wave of `occ` warps per SM allows; `busiest` is
+// the segments on the SM with the most resident workers (workers spread evenly over the SMs).
+struct SegSplit {
+  int64_t k, workers, busiest;
+};
+inline SegSplit seg_split(int64_t nseg, int occ, int num_sms) {
+  const int64_t slots = (int64_t)(occ > 0 ? occ : 1) * num_sms;
+  const int64_t k = (nseg + slots - 1) / slots;
+  const int64_t workers = (nseg + k - 1) / k;
+  return {k, workers, (workers + num_sms - 1) / num_sms * k};
+}
+
 template <typename T, int D>
 cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a, int num_sms,
                             cudaStream_t stream, int* grid, DecodePlan* plan) {
   constexpr int AK = KVC_DEC_SEG_KPT, AS = KVC_DEC_SEG_STAGES;
   constexpr int BK = KVC_DEC_SEG2_KPT, BS = KVC_DEC_SEG2_STAGES;
   constexpr int TK = KVC_DEC_STREAM_KPT, TS = KVC_DEC_STREAM_STAGES;
-  // One warp per (sequence, head) segment when the segments are balanced (longest within 1.3x of
-  // the mean) and all fit one wave of resident warps: no split-K partials.  The wider pipeline
-  // shape is tried first.  Otherwise the rows are split evenly over a full wave (stream-K).
+  // Balanced segments (longest within 1.3x of the mean) are never split, so no warp writes split-K
+  // partials or waits on a combine: one warp per (sequence, head) segment when a wave of resident
+  // warps holds them all (the wider pipeline shape first), else k consecutive whole segments per
+  // warp, with the shape and k that put the fewest segments on the busiest SM.  Otherwise the
+  // rows are split evenly over a full wave (stream-K).
   const int64_t nseg = (int64_t)g.b * g.H;
   const bool balanced = a.n_segments > 0 && nseg <= kMaxDecodeWorkers && 10 * a.max_segment * a.n_segments <= 13 * a.R;
   cudaError_t e;
   if (balanced) {
-    int occ = 0;
-    e = decode_occupancy<T, D, AK, AS>(&occ);
+    int occ_a = 0, occ_b = 0;
+    e = decode_occupancy<T, D, AK, AS>(&occ_a);
+    if (e == cudaSuccess) e = decode_occupancy<T, D, BK, BS>(&occ_b);
     if (e != cudaSuccess) return e;
-    if (nseg <= (int64_t)occ * num_sms) {
+    if (nseg <= (int64_t)occ_a * num_sms) {
       *plan = {1, (int)nseg, AK * Lanes<D>::RPI, AS};
-      return launch_decode_cfg<T, D, AK, AS>(g, st, buf, a, nseg, true, stream, grid);
+      return launch_decode_cfg<T, D, AK, AS>(g, st, buf, a, nseg, 1, stream, grid);
     }
-    e = decode_occupancy<T, D, BK, BS>(&occ);
-    if (e != cudaSuccess) return e;
-    if (nseg <= (int64_t)occ * num_sms) {
+    if (nseg <= (int64_t)occ_b * num_sms) {
       *plan = {2, (int)nseg, BK * Lanes<D>::RPI, BS};
-      return launch_decode_cfg<T, D, BK, BS>(g, st, buf, a, nseg, true, stream, grid);
+      return launch_decode_cfg<T, D, BK, BS>(g, st, buf, a, nseg, 1, stream, grid);
     }
+    const SegSplit sa = seg_split(nseg, occ_a, num_sms), sb = seg_split(nseg, occ_b, num_sms);
+    if (sa.busiest <= sb.busiest) {
+      *plan = {3, (int)sa.workers, AK * Lanes<D>::RPI, AS};
+      return launch_decode_cfg<T, D, AK, AS>(g, st, buf, a, sa.workers, sa.k, stream, grid);
+    }
+    *plan = {3, (int)sb.workers, BK * Lanes<D>::RPI, BS};
+    return launch_decode_cfg<T, D, BK, BS>(g, st, buf, a, sb.workers, sb.k, stream, grid);
   }
   int occ = 0;
   e = decode_occupancy<T, D, TK, TS>(&occ);
@@ -833,7 +857,7 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   if (NW > kMaxDecodeWorkers) NW = kMaxDecodeWorkers;
   if (NW < 1) NW = 1;
   *plan = {0, (int)NW, TK * Lanes<D>::RPI, TS};
-  return launch_decode_cfg<T, D, TK, TS>(g, st, buf, a, NW, false, stream, grid);
+  return launch_decode_cfg<T, D, TK, TS>(g, st, buf, a, NW, 0, stream, grid);
 }
 
 template <typename T, int D>

@@ -203,6 +203,7 @@ def test_launch_counter_counts_kernels():
 def _mode_workloads():
     sms = torch.cuda.get_device_properties(0).multi_processor_count if torch.cuda.is_available() else 152
     b_narrow = (5 * sms + 31) // 32  # more segments than one wave of the wide pipeline holds (4 warps/SM at d=64)
+    b_multi = (10 * sms + 31) // 32  # more than one wave of the narrow pipeline holds (8 warps/SM at d=64)
     long_short = dataclasses.replace(wl.opt13b(b=2, L=64, M=1), name="long-short")
     k_long, s_long = wl.block_kinds(5000, 32)
     k_short, s_short = wl.block_kinds(70, 8)
@@ -210,14 +211,15 @@ def _mode_workloads():
     long_short.prompt_spans = [s_long, s_short]
     return [("wide", wl.opt13b(b=3, L=640, M=1), 1),
             ("narrow", wl.opt13b(b=b_narrow, L=192, M=1), 2),
+            ("several segments per warp", wl.opt13b(b=b_multi, L=192, M=1), 3),
             ("stream-k", long_short, 0),
             ("ragged stream-k", wl.ragged(b=40, lmin=64, lmax=1500, M=1, steps=4), 0)]
 
 
 @pytest.mark.parametrize("name,w,mode", _mode_workloads(), ids=lambda x: x if isinstance(x, str) else "")
 def test_every_scheduling_mode(name, w, mode):
-    # each way of dividing the decode work (one warp per segment, wide or narrow pipeline; stream-K
-    # with split segments) must agree with the oracle
+    # each way of dividing the decode work (one warp per segment, wide or narrow pipeline; several
+    # whole segments per warp; stream-K with split segments) must agree with the oracle
     run, _ = run_workload(w, steps=2, check_steps={0, 1}, seqs=None)
     plan = run.cache.last_decode_plan
     assert plan["mode"] == mode, plan
