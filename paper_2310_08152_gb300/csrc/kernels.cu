@@ -638,6 +638,7 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
     const bool seg_done = (r0 + n == ci.Lc);
     ci.advance(n, p.P, H);
     ++t;
+    bool refilled = false;
     if (seg_done || ci.done()) {
       // ------------------------- piece end: merge the row groups -------------------------
       float M = m;
@@ -684,6 +685,14 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
             pp[0] = M;
             pp[1] = Ls;
           }
+          // the stage is read: refill it before the fence and the arrival, which wait on memory
+          __syncwarp();
+          if (lane == 0 && !ii.done()) {
+            fence_proxy_async_smem();
+            issue(stage);
+            ++issued;
+          }
+          refilled = true;
           __threadfence();
           __syncwarp();
           const int64_t Lc = p.P[s + 1] - p.P[s];
@@ -726,7 +735,7 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
       piece_start = true;
     }
     // refill the stage just consumed
-    if (lane == 0 && !dead && !ii.done()) {
+    if (lane == 0 && !dead && !refilled && !ii.done()) {
       fence_proxy_async_smem();
       issue(stage);
       ++issued;
