@@ -203,7 +203,9 @@ def test_launch_counter_counts_kernels():
 def _mode_workloads():
     sms = torch.cuda.get_device_properties(0).multi_processor_count if torch.cuda.is_available() else 152
     b_narrow = (5 * sms + 31) // 32  # more segments than one wave of the wide pipeline holds (4 warps/SM at d=64)
-    b_multi = (10 * sms + 31) // 32  # more than one wave of the narrow pipeline holds (8 warps/SM at d=64)
+    # more segments than one wave of the narrow pipeline holds (8 warps/SM at d=64), and a count that
+    # k does not divide, so the last worker takes fewer segments
+    b_multi = (10 * sms + 31) // 32 + 1
     long_short = dataclasses.replace(wl.opt13b(b=2, L=64, M=1), name="long-short")
     k_long, s_long = wl.block_kinds(5000, 32)
     k_short, s_short = wl.block_kinds(70, 8)
