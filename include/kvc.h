@@ -186,6 +186,7 @@ const kvc_book* kvc_get_book(const kvc_cache* cache);
  *   layer == -1: all layers at once; k, v are device [M][N][H][d_head] with N = sum(n_new).
  *   layer == 0 .. M-1: one layer, k, v are [N][H][d_head]; layer 0 starts a new batch of tokens
  *     (n_new, pos, kinds used); layers 1.. must follow in order and ignore n_new/pos/kinds.
+ * k and v are 16-byte aligned (else KVC_ERR_INVALID_ARG).
  * n_new[b], pos[N], kinds[N] are host arrays (sequence-major).  With rotary_dim > 0, K is rotated
  * at its position before it is stored.  A <CL> row is stored and skipped by later queries until
  * its span is freed (paper policy).  Errors: KVC_ERR_CAPACITY, KVC_ERR_SPAN, KVC_ERR_STATE. */

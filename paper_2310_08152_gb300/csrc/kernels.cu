@@ -14,6 +14,7 @@
 //
 // No tensor cores: one query per (sequence, head) makes decode a GEMV (1 flop per byte read), far
 // below any tensor-core ridge; the kernels are bound by HBM bandwidth.
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -109,6 +110,144 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(Geometry g, Stat
       buf.pos[st.off[tp.s] + tp.row] = tp.pos;
       buf.orig[st.off[tp.s] + tp.row] = tp.orig;
     }
+  }
+}
+
+// a1 through TMA, for calls with at least one (layer, token) unit per SM.  A warp is a worker with
+// a ring of kAppStages slots; a slot holds one unit's K and V rows of every head, which lie
+// contiguously in the input.  Lane 0 brings a unit in with two bulk copies, kAppLag units ahead,
+// and writes it out with two tensor stores over the sequence's 4-D map {d, row, head, layer}: the
+// box {d, 1, H, 1} sends each head's row to its own (layer, K/V, head) stream.  With RoPE the warp
+// rotates K in shared memory in between.  No registers hold the rows, so several units per warp
+// and several warps per SM are in flight.
+constexpr int kAppStages = 4;
+constexpr int kAppLag = 2;
+static_assert(kAppLag >= 1 && kAppLag < kAppStages, "loads run ahead of stores by fewer units than slots");
+
+__host__ __device__ constexpr uint32_t app_slot_bytes(int H, int D) { return ((uint32_t)H * D * 2 + 127u) / 128u * 128u; }
+inline size_t app_smem_bytes(int H, int D, int rot) {
+  return (size_t)kAppStages * 2 * app_slot_bytes(H, D) + 8 * (size_t)kAppStages + 8 * (size_t)(rot > 1 ? rot / 2 : 1);
+}
+
+__device__ __forceinline__ void tma_store_4d(const CUtensorMap* map, const void* src, int x, int y, int z, int w) {
+  asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%1, %2, %3, %4}], [%5];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z), "r"(w), "r"(smem_addr(src))
+               : "memory");
+}
+__device__ __forceinline__ void app_bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// waits until at most N of this thread's bulk groups are still reading shared memory
+template <int N>
+__device__ __forceinline__ void app_bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void app_bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+template <typename T, int D>
+__global__ void __launch_bounds__(32, 1) append_tma_kernel(Geometry g, Static st, Buffers buf,
+                                                           const TokPlan* __restrict__ plan, int64_t ntok, int64_t n_in,
+                                                           int m0, int n_layers, int write_meta,
+                                                           const uint16_t* __restrict__ k_in,
+                                                           const uint16_t* __restrict__ v_in,
+                                                           const CUtensorMap* __restrict__ maps,
+                                                           unsigned long long limit_ns) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  const int lane = threadIdx.x;
+  const int H = g.H;
+  const uint32_t ub = (uint32_t)H * D * 2;  // bytes of one unit's K (or V) rows
+  const uint32_t slot = app_slot_bytes(H, D);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kAppStages * 2 * slot);
+  float2* cs = reinterpret_cast<float2*>(full + kAppStages);  // (cos, sin) per rotated pair, one unit
+  const int hp = g.rot / 2;   // rotated pairs per head
+  const int hv = g.rot / 16;  // 16-byte vector pairs per head
+  const int64_t n_units = (int64_t)n_layers * ntok;
+  const int64_t w = blockIdx.x, NW = gridDim.x;
+  const int64_t n_my = w < n_units ? (n_units - 1 - w) / NW + 1 : 0;  // units w, w + NW, ...
+  if (lane == 0) {
+#pragma unroll
+    for (int i = 0; i < kAppStages; ++i) mbar_init(&full[i], 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+  int64_t loaded = 0;  // units whose copies lane 0 has issued
+  int64_t k = 0;
+  for (; k < n_my + kAppLag; ++k) {
+    if (k < n_my && lane == 0) {
+      const int sl = (int)(k % kAppStages);
+      // the slot's previous unit (k - kAppStages) has been read out by its stores: stores of at most
+      // kAppStages - 1 - kAppLag newer units may still be reading
+      if (k >= kAppStages) app_bulk_wait_read<kAppStages - 1 - kAppLag>();
+      fence_proxy_async_smem();  // after the generic accesses (rotation) to the slot's previous unit
+      const int64_t u = w + k * NW;
+      const int l = (int)(u / ntok);
+      const int64_t src = ((int64_t)l * n_in + plan[u - (int64_t)l * ntok].in_tok) * H * D;
+      unsigned char* d0 = smem + (size_t)sl * 2 * slot;
+      mbar_arrive_expect_tx(&full[sl], 2 * ub);
+      bulk_g2s(d0, k_in + src, ub, &full[sl]);
+      bulk_g2s(d0 + slot, v_in + src, ub, &full[sl]);
+      loaded = k + 1;
+    }
+    const int64_t j = k - kAppLag;
+    if (j < 0 || j >= n_my) continue;
+    const int sl = (int)(j % kAppStages);
+    const int64_t u = w + j * NW;
+    const int l = (int)(u / ntok);
+    const TokPlan tp = plan[u - (int64_t)l * ntok];
+    if (hv > 0) {
+      __syncwarp();  // the previous unit's rotations are done with the table
+      for (int i = lane; i < hp; i += 32) {
+        float sn, c;
+        rope_sincos(tp.pos, st.rope_g[i], &sn, &c);
+        cs[i] = make_float2(c, sn);
+      }
+      __syncwarp();
+    }
+    if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(&full[sl], (uint32_t)(j / kAppStages) & 1, limit_ns))) {
+      if (lane == 0) atomicOr(buf.status, STATUS_TIMEOUT);
+      break;
+    }
+    unsigned char* ks = smem + (size_t)sl * 2 * slot;
+    if (hv > 0) {
+      for (int it = lane; it < H * hv; it += 32) {
+        const int h = it / hv, vec = it - h * hv;
+        uint4* qa = reinterpret_cast<uint4*>(ks + ((size_t)h * D + vec * 8) * 2);
+        uint4* qb = reinterpret_cast<uint4*>(ks + ((size_t)h * D + (vec + hv) * 8) * 2);
+        const uint4 a = *qa, b = *qb;
+        const uint16_t* xa = reinterpret_cast<const uint16_t*>(&a);
+        const uint16_t* xb = reinterpret_cast<const uint16_t*>(&b);
+        uint4 ya, yb;
+        uint16_t* pa = reinterpret_cast<uint16_t*>(&ya);
+        uint16_t* pb = reinterpret_cast<uint16_t*>(&yb);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float2 r = cs[vec * 8 + e];
+          const float x1 = T::f1(xa[e]), x2 = T::f1(xb[e]);
+          pa[e] = T::r(x1 * r.x - x2 * r.y);
+          pb[e] = T::r(x2 * r.x + x1 * r.y);
+        }
+        *qa = ya;
+        *qb = yb;
+      }
+      fence_proxy_async_smem();  // the rotated rows, before the tensor store reads them
+      __syncwarp();
+    }
+    if (lane == 0) {
+      tma_store_4d(maps + tp.s, ks, 0, tp.row, 0, m0 + l);
+      tma_store_4d(maps + g.b + tp.s, ks + slot, 0, tp.row, 0, m0 + l);
+      app_bulk_commit();
+      if (write_meta && l == 0) {
+        buf.pos[st.off[tp.s] + tp.row] = tp.pos;
+        buf.orig[st.off[tp.s] + tp.row] = tp.orig;
+      }
+    }
+  }
+  if (lane == 0) {
+    if (k < n_my + kAppLag) {
+      // gave up waiting: let the copies still in flight land (bounded) before the slots go away
+      for (int64_t x = (k - kAppLag > 0 ? k - kAppLag : 0); x < loaded; ++x)
+        (void)mbar_wait_bounded(&full[x % kAppStages], (uint32_t)(x / kAppStages) & 1, limit_ns);
+    }
+    app_bulk_wait_all();  // every tensor store has completed
   }
 }
 
@@ -872,9 +1011,34 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
 template <typename T, int D>
 cudaError_t launch_append_t(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t ntok,
                             int64_t n_in, int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
-                            cudaStream_t stream) {
+                            const void* maps, int num_sms, unsigned long long limit_ns, cudaStream_t stream) {
+  const int64_t n_units = (int64_t)n_layers * ntok;
+  const size_t smem = app_smem_bytes(g.H, D, g.rot);
+  if (maps != nullptr && num_sms > 0 && n_units >= num_sms && smem <= 200 * 1024) {
+    // TMA ring workers, as many one-warp CTAs as fit (capped by the units)
+    static size_t smem_set = 0;  // per instantiation: the dynamic shared memory opted into so far
+    static size_t occ_for = 0;
+    static int occ = 0;
+    cudaError_t e = cudaSuccess;
+    if (smem > smem_set) {
+      e = cudaFuncSetAttribute(append_tma_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return e;
+      smem_set = smem;
+    }
+    if (occ_for != smem) {
+      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, append_tma_kernel<T, D>, 32, smem);
+      if (e != cudaSuccess) return e;
+      occ_for = smem;
+    }
+    int64_t grid = (int64_t)(occ > 0 ? occ : 1) * num_sms;
+    if (grid > n_units) grid = n_units;
+    append_tma_kernel<T, D><<<(unsigned)grid, 32, smem, stream>>>(
+        g, st, buf, plan, ntok, n_in, m0, n_layers, write_meta ? 1 : 0, static_cast<const uint16_t*>(k_in),
+        static_cast<const uint16_t*>(v_in), static_cast<const CUtensorMap*>(maps), limit_ns);
+    return cudaGetLastError();
+  }
   // one (layer, token) unit per block at a time; enough blocks for every SM several times over
-  int64_t blocks = (int64_t)n_layers * ntok;
+  int64_t blocks = n_units;
   if (blocks > kAppendMaxBlocks) blocks = kAppendMaxBlocks;
   if (blocks < 1) blocks = 1;
   append_kernel<T, D><<<(unsigned)blocks, kAppendThreads, 0, stream>>>(g, st, buf, plan, ntok, n_in, m0, n_layers, write_meta ? 1 : 0,
@@ -905,12 +1069,14 @@ bool dhead_supported(int D) { return D == 64 || D == 80 || D == 96 || D == 128; 
 
 cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t n_plan,
                           int64_t n_in, int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
-                          cudaStream_t stream) {
+                          const void* maps, int num_sms, unsigned long long limit_ns, cudaStream_t stream) {
   return by_dhead(g.D, [&](auto dc) {
     constexpr int D = decltype(dc)::value;
     if (g.dtype == 1)
-      return launch_append_t<BF16T, D>(g, st, buf, plan, n_plan, n_in, m0, n_layers, write_meta, k_in, v_in, stream);
-    return launch_append_t<F16T, D>(g, st, buf, plan, n_plan, n_in, m0, n_layers, write_meta, k_in, v_in, stream);
+      return launch_append_t<BF16T, D>(g, st, buf, plan, n_plan, n_in, m0, n_layers, write_meta, k_in, v_in, maps,
+                                       num_sms, limit_ns, stream);
+    return launch_append_t<F16T, D>(g, st, buf, plan, n_plan, n_in, m0, n_layers, write_meta, k_in, v_in, maps,
+                                    num_sms, limit_ns, stream);
   });
 }
 

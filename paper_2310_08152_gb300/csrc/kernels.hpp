@@ -57,10 +57,21 @@ constexpr int kMaxDecodeWorkers = 8192;
 
 bool dhead_supported(int D);
 
-// Writes the n_plan stored tokens of a call whose inputs hold n_in tokens per layer.
+// Writes the n_plan stored tokens of a call whose inputs hold n_in tokens per layer (k_in, v_in
+// 16-byte aligned).  maps: the device copy of encode_append_maps' output, or NULL; with it, calls of
+// at least num_sms (layer, token) units go through the TMA kernel, whose bounded waits give up
+// after limit_ns.
 cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& buf, const TokPlan* plan, int64_t n_plan,
                           int64_t n_in, int m0, int n_layers, bool write_meta, const void* k_in, const void* v_in,
-                          cudaStream_t stream);
+                          const void* maps, int num_sms, unsigned long long limit_ns, cudaStream_t stream);
+// Bytes of encode_append_maps' output: a 128-byte TMA descriptor per (K/V, sequence).
+inline size_t append_maps_bytes(int b) { return 2 * 128 * (size_t)b; }
+// Encodes, per sequence s, 4-D TMA descriptors over the K and then the V planes: dims {D, cap[s],
+// H, M} from row seq_row0[s] of layer 0's plane, strides (D, cap[s] D, H C D) elements, box
+// {D, 1, H, 1}: one (layer, token)'s rows of every head.  seq_row0 and cap are host arrays; out is
+// host memory of append_maps_bytes(b).  cudaErrorNotSupported where a box cannot hold H heads.
+cudaError_t encode_append_maps(const Geometry& g, const Buffers& buf, const int64_t* seq_row0, const int32_t* cap,
+                               unsigned char* out);
 
 cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& buf, const AffSeq* aff, int n_aff,
                            const int32_t* ranges, int32_t* src_map, cudaStream_t stream, int* launched);

@@ -51,6 +51,7 @@ struct WsLayout {
   size_t st_cap = 0;     // int32 [b]
   size_t st_off = 0;     // int64 [b]
   size_t st_rope = 0;    // float2 [max(1, rot/2)]
+  size_t amaps = 0;      // TMA descriptors of the append kernel: [K/V][b] x 128 bytes
   size_t dyn = 0;        // [DState b][int64 P b+1][payload]
   size_t dyn_P = 0;      // offset of P inside dyn
   size_t dyn_payload = 0;  // offset of the payload inside dyn
@@ -80,6 +81,7 @@ WsLayout ws_layout(int b, int H, int D, int rot, int64_t C) {
   L.st_cap = take(4 * (size_t)b);
   L.st_off = take(8 * (size_t)b);
   L.st_rope = take(8 * (size_t)std::max(1, rot / 2));
+  L.amaps = take(kvc::append_maps_bytes(b));
   L.dyn_P = align_up(sizeof(kvc::DState) * (size_t)b, 16);
   L.dyn_payload = align_up(L.dyn_P + 8 * (size_t)(b + 1), 16);
   const size_t tok = sizeof(kvc::TokPlan) * (size_t)C;
@@ -235,6 +237,7 @@ struct kvc_cache {
   int64_t pre_tiles = 0;
   int pre_ctas = 0;
   kvc::PrefillMaps maps;
+  bool amaps_ok = false;  // the append kernel's TMA descriptors are in the workspace
 
   kvc_cache(const kvc_config& c, int64_t C_)
       : cfg(c), C(C_), bk(c.b, (kvc::Policy)c.policy, c.seq_capacity, (double)c.local_ratio) {
@@ -290,7 +293,7 @@ struct kvc_cache {
     }
     e = cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
-    e = ring.init(2 * ws.dyn_bytes + ws.pre_bytes + 2 * ws.st_rope + 65536);
+    e = ring.init(2 * ws.dyn_bytes + ws.pre_bytes + 2 * ws.st_rope + kvc::append_maps_bytes(cfg.b) + 65536);
     if (e != cudaSuccess) return cuda_fail(e, "cudaHostAlloc (staging ring)");
     // static tables
     const int b = cfg.b, half = std::max(1, cfg.rotary_dim / 2);
@@ -316,6 +319,22 @@ struct kvc_cache {
     }
     e = ring.commit(wsp(ws.st_row0), st_bytes, stream);
     if (e != cudaSuccess) return cuda_fail(e, "upload static tables");
+    // the append kernel's TMA descriptors (64-byte aligned in the workspace); without them (a box
+    // cannot hold H heads) appends take the kernel that copies through registers
+    amaps_ok = false;
+    if ((reinterpret_cast<uintptr_t>(wsp(ws.amaps)) & 63) == 0) {
+      std::vector<int32_t> cap32(cap.begin(), cap.end());
+      std::vector<int64_t> row0h(b);
+      for (int s = 0; s < b; ++s) row0h[s] = (int64_t)cfg.H * off[s];
+      const size_t mb = kvc::append_maps_bytes(b);
+      unsigned char* hm = ring.reserve(mb, &e);
+      if (!hm) return e != cudaSuccess ? cuda_fail(e, "staging") : fail(KVC_ERR_INVALID_ARG, "descriptors exceed ring");
+      if (kvc::encode_append_maps(geom(), bufs(), row0h.data(), cap32.data(), hm) == cudaSuccess) {
+        e = ring.commit(wsp(ws.amaps), mb, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "upload append descriptors");
+        amaps_ok = true;
+      }
+    }
     e = cudaMemsetAsync(wsp(ws.hdr), 0, 256, stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(wsp(ws.counters), 0, 4 * (size_t)cfg.b * cfg.H, stream);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
@@ -595,6 +614,8 @@ static kvc_status append_impl(kvc_cache* c, int layer, const void* k, const void
   const int M = c->cfg.M;
   if (layer < -1 || layer >= M) return fail(KVC_ERR_INVALID_ARG, "layer %d out of range [-1, %d)", layer, M);
   if (!k || !v) return fail(KVC_ERR_INVALID_ARG, "k/v are NULL");
+  if ((reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(v)) & 15)
+    return fail(KVC_ERR_INVALID_ARG, "k and v must be 16-byte aligned");
   const bool starts = layer <= 0;
   if (starts) {
     if (c->layers_done != M)
@@ -670,7 +691,8 @@ static kvc_status append_impl(kvc_cache* c, int layer, const void* k, const void
   if (c->batch_ntok > 0) {
     const kvc::TokPlan* plan = reinterpret_cast<const kvc::TokPlan*>(c->wsp(c->ws.dyn + c->ws.dyn_payload));
     cudaError_t e = kvc::launch_append(g, c->stat(), c->bufs(), plan, c->batch_ntok, c->batch_nin, m0, nl, m0 == 0, k,
-                                       v, stream);
+                                       v, c->amaps_ok ? c->wsp(c->ws.amaps) : nullptr, c->num_sms, 2000000000ull,
+                                       stream);
     if (e != cudaSuccess) return cuda_fail(e, "append kernel");
     c->launches += 1;
     c->last_was_decode = false;

@@ -983,16 +983,45 @@ cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int6
 
 }  // namespace
 
-cudaError_t encode_prefill_maps(const Geometry& g, const Buffers& buf, PrefillMaps* maps) {
-  static_assert(sizeof(CUtensorMap) == sizeof(maps->k), "tensor map size");
+static cudaError_t load_encoder() {
   std::call_once(g_encode_once, [] {
     cudaDriverEntryPointQueryResult q;
     g_encode_err = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", reinterpret_cast<void**>(&g_encode),
                                                     12000, cudaEnableDefault, &q);
     if (g_encode_err == cudaSuccess && q != cudaDriverEntryPointSuccess) g_encode_err = cudaErrorNotSupported;
   });
-  if (g_encode_err != cudaSuccess) return g_encode_err;
-  cudaError_t e = encode_plane(g, buf.k, maps->k);
+  return g_encode_err;
+}
+
+cudaError_t encode_append_maps(const Geometry& g, const Buffers& buf, const int64_t* seq_row0, const int32_t* cap,
+                               unsigned char* out) {
+  static_assert(sizeof(CUtensorMap) == 128, "tensor map size");
+  if (g.H > 256 || g.D > 256) return cudaErrorNotSupported;  // box dimensions hold at most 256 elements
+  cudaError_t e = load_encoder();
+  if (e != cudaSuccess) return e;
+  for (int kv = 0; kv < 2; ++kv) {
+    for (int s = 0; s < g.b; ++s) {
+      uint16_t* base = (kv ? buf.v : buf.k) + seq_row0[s] * g.D;
+      cuuint64_t dims[4] = {(cuuint64_t)g.D, (cuuint64_t)cap[s], (cuuint64_t)g.H, (cuuint64_t)g.M};
+      cuuint64_t strides[3] = {(cuuint64_t)g.D * 2, (cuuint64_t)cap[s] * g.D * 2, (cuuint64_t)g.H * g.C * g.D * 2};
+      cuuint32_t box[4] = {(cuuint32_t)g.D, 1, (cuuint32_t)g.H, 1};
+      cuuint32_t elem[4] = {1, 1, 1, 1};
+      CUtensorMap m;
+      const CUresult r = g_encode(&m, CU_TENSOR_MAP_DATA_TYPE_UINT16, 4, base, dims, strides, box, elem,
+                                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                                  CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+      std::memcpy(out + 128 * ((size_t)kv * g.b + s), &m, sizeof m);
+    }
+  }
+  return cudaSuccess;
+}
+
+cudaError_t encode_prefill_maps(const Geometry& g, const Buffers& buf, PrefillMaps* maps) {
+  static_assert(sizeof(CUtensorMap) == sizeof(maps->k), "tensor map size");
+  cudaError_t e = load_encoder();
+  if (e != cudaSuccess) return e;
+  e = encode_plane(g, buf.k, maps->k);
   if (e == cudaSuccess) e = encode_plane(g, buf.v, maps->v);
   maps->ready = e == cudaSuccess;
   return e;
