@@ -206,6 +206,7 @@ def _mode_workloads():
     # more segments than one wave of the narrow pipeline holds (8 warps/SM at d=64), and a count that
     # k does not divide, so the last worker takes fewer segments
     b_multi = (10 * sms + 31) // 32 + 1
+    b_multi80 = (9 * sms) // 32 + 1  # d=80 rotary: beyond a wave of the narrow pipeline (7 warps/SM)
     long_short = dataclasses.replace(wl.opt13b(b=2, L=64, M=1), name="long-short")
     k_long, s_long = wl.block_kinds(5000, 32)
     k_short, s_short = wl.block_kinds(70, 8)
@@ -214,6 +215,7 @@ def _mode_workloads():
     return [("wide", wl.opt13b(b=3, L=640, M=1), 1),
             ("narrow", wl.opt13b(b=b_narrow, L=192, M=1), 2),
             ("several segments per warp", wl.opt13b(b=b_multi, L=192, M=1), 3),
+            ("several segments per warp, d=80 rotary", wl.rope3b(32, b=b_multi80, L=192, M=1), 3),
             ("stream-k", long_short, 0),
             ("ragged stream-k", wl.ragged(b=40, lmin=64, lmax=1500, M=1, steps=4), 0)]
 
