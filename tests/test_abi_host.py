@@ -217,6 +217,11 @@ def test_cache_validates_before_any_device_work():
         assert L.kvc_append(h, -1, fake, fake, big.ctypes.data, np.zeros(17, np.int32).ctypes.data,
                             np.zeros(17, np.uint8).ctypes.data, None) == 3
         assert L.kvc_append(h, 1, fake, fake, None, None, None, None) == 5   # layer 1 before layer 0
+        # inputs the bulk copies cannot start from: not 16-byte aligned
+        assert L.kvc_append(h, -1, fake + 8, fake, n_new.ctypes.data, pos.ctypes.data, np.uint8([0, 0]).ctypes.data,
+                            None) == 1
+        assert L.kvc_append(h, 0, fake, fake + 2, n_new.ctypes.data, pos.ctypes.data, np.uint8([0, 0]).ctypes.data,
+                            None) == 1
         assert L.kvc_decode_attention(h, 0, fake, ctypes.c_float(0.125), fake, None) == 5  # nothing appended
         assert L.kvc_decode_attention(h, 9, fake, ctypes.c_float(0.125), fake, None) == 1
         n = 2 * 4 * 64
