@@ -2,6 +2,7 @@
 seconds: several tiles per segment, split segments, ragged tails, every step kind (normal, <CL>
 query, open-span queries, <CR> query, compaction right after it), both policies, every built d_head."""
 import dataclasses
+import math
 
 import numpy as np
 import pytest
@@ -75,6 +76,15 @@ def test_keep_cl_policy():
 def test_every_built_head_dim(d, dtype):
     w = dataclasses.replace(wl.opt13b(b=2, L=448, M=2), d=d, dtype=dtype, name=f"d{d}-{dtype}")
     run_workload(w, steps=34, check_steps={0, 1, 31, 32, 33})
+
+
+@pytest.mark.parametrize("d,rot", [(96, 96), (128, 64)])
+def test_rope_other_head_dims(d, rot):
+    # rotation of 6 / 4 vector pairs per head (d_head 96 whole, 128 half), four lanes per row
+    w = dataclasses.replace(wl.rope3b(32, b=2, L=384, M=1), d=d, rotary_dim=rot, scale=1.0 / math.sqrt(d),
+                            name=f"rope-d{d}-r{rot}")
+    run, _ = run_workload(w, steps=3)
+    check_rows(run, 3, 0, 0, [1], check_k=False)  # K is stored rotated
 
 
 def test_rope_partial_rotary_dim():

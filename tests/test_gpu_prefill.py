@@ -4,6 +4,7 @@ block with the spans each block closed freed in between, ragged lengths and quer
 mid-tile, RoPE (full and partial rotary dimension, f16 and bf16), both policies, every built d_head
 and both 16-bit types."""
 import dataclasses
+import math
 
 import numpy as np
 import pytest
@@ -176,6 +177,14 @@ def test_prefill_rope_bf16():
     # the query rotation rounded to bf16 (held to eight times the f16 bound)
     w = dataclasses.replace(wl.rope3b(32, b=2, L=400, M=1), dtype="bf16", name="rope-bf16")
     run_prefill(w, 0, layers=[0], heads=[0, 31])
+
+
+@pytest.mark.parametrize("d,rot", [(96, 96), (128, 64)])
+def test_prefill_rope_other_head_dims(d, rot):
+    # one CTA per SM (d_head 96 / 128) with the query rotated over 48 / 32 pairs
+    w = dataclasses.replace(wl.rope3b(32, b=2, L=384, M=1), d=d, rotary_dim=rot, scale=1.0 / math.sqrt(d),
+                            name=f"rope-d{d}-r{rot}")
+    run_prefill(w, 0, layers=[0], heads=[3, 30])
 
 
 def test_prefill_rope_partial_rotary_dim():
