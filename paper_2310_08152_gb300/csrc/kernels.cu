@@ -22,6 +22,7 @@
 #include <cmath>
 #include <cstdint>
 #include <mutex>
+#include <vector>
 
 #include "device_common.cuh"
 #include "kernels.hpp"
@@ -249,6 +250,41 @@ __global__ void __launch_bounds__(32, 1) append_tma_kernel(Geometry g, Static st
     }
     app_bulk_wait_all();  // every tensor store has completed
   }
+}
+
+// Resident one-warp CTAs of append_tma_kernel per SM for `smem` bytes of dynamic shared memory on
+// the current device; the opt-in to that size is made per device as needed.
+template <typename T, int D>
+cudaError_t append_tma_occupancy(size_t smem, int* occ_out) {
+  struct Seen {
+    size_t smem;
+    int occ;
+  };
+  static std::mutex mu;
+  static size_t opted[64] = {};
+  static std::vector<Seen> seen[64];
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  for (const Seen& x : seen[dev])
+    if (x.smem == smem) {
+      *occ_out = x.occ;
+      return cudaSuccess;
+    }
+  if (smem > opted[dev]) {
+    e = cudaFuncSetAttribute(append_tma_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    opted[dev] = smem;
+  }
+  int o = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, append_tma_kernel<T, D>, 32, smem);
+  if (e != cudaSuccess) return e;
+  if (o < 1) o = 1;
+  seen[dev].push_back({smem, o});
+  *occ_out = o;
+  return cudaSuccess;
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -1016,21 +1052,10 @@ cudaError_t launch_append_t(const Geometry& g, const Static& st, const Buffers& 
   const size_t smem = app_smem_bytes(g.H, D, g.rot);
   if (maps != nullptr && num_sms > 0 && n_units >= num_sms && smem <= 200 * 1024) {
     // TMA ring workers, as many one-warp CTAs as fit (capped by the units)
-    static size_t smem_set = 0;  // per instantiation: the dynamic shared memory opted into so far
-    static size_t occ_for = 0;
-    static int occ = 0;
-    cudaError_t e = cudaSuccess;
-    if (smem > smem_set) {
-      e = cudaFuncSetAttribute(append_tma_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      if (e != cudaSuccess) return e;
-      smem_set = smem;
-    }
-    if (occ_for != smem) {
-      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, append_tma_kernel<T, D>, 32, smem);
-      if (e != cudaSuccess) return e;
-      occ_for = smem;
-    }
-    int64_t grid = (int64_t)(occ > 0 ? occ : 1) * num_sms;
+    int occ = 0;
+    const cudaError_t e = append_tma_occupancy<T, D>(smem, &occ);
+    if (e != cudaSuccess) return e;
+    int64_t grid = (int64_t)occ * num_sms;
     if (grid > n_units) grid = n_units;
     append_tma_kernel<T, D><<<(unsigned)grid, 32, smem, stream>>>(
         g, st, buf, plan, ntok, n_in, m0, n_layers, write_meta ? 1 : 0, static_cast<const uint16_t*>(k_in),

@@ -946,8 +946,16 @@ cudaError_t encode_plane(const Geometry& g, void* base, unsigned char* out) {
 
 template <typename T, int D>
 cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int64_t grid, cudaStream_t stream) {
-  static bool attr_set = false;  // per instantiation; setting it twice is harmless
-  if (!attr_set) {
+  static std::mutex mu;
+  static bool attr_set[64] = {};  // per device: the shared-memory opt-in and the register check
+  int dev = 0;
+  {
+    const cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!attr_set[dev]) {
     const cudaError_t e = cudaFuncSetAttribute(prefill_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)PfCfg<D>::SMEM);
     if (e != cudaSuccess) return e;
@@ -959,7 +967,7 @@ cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int6
       if (e2 != cudaSuccess) return e2;
       if (fa.numRegs != PfCfg<D>::REG_LAUNCH) return cudaErrorInvalidConfiguration;
     }
-    attr_set = true;
+    attr_set[dev] = true;
   }
   CUtensorMap mk, mv, mo;
   std::memcpy(&mk, maps.k, sizeof mk);
