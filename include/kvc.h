@@ -76,6 +76,8 @@ typedef enum {
   KVC_POLICY_LOCAL = 2
 } kvc_policy;
 
+/* A static, NUL-terminated description of status `s` ("ok", "span error", ...; a fixed text for a
+ * value outside the enum).  Host only, never fails; the caller does not free it. */
 const char* kvc_status_string(kvc_status s);
 /* Detail of the last error returned on this thread ("" if none).  Valid until the next call. */
 const char* kvc_last_error(void);
