@@ -45,8 +45,15 @@ constexpr int kItemRing = 4;
 // Shared-memory geometry for head dimension D.  Q, K and V tiles are [128 rows][D] split into
 // column subtiles of SW bytes per row, the widest swizzle (128 / 64 / 32 bytes) that divides a row;
 // each subtile is the canonical K-major (Q, K) or MN-major (V) layout of that swizzle.
-template <int D>
+//
+// SPLIT (bf16): the rotated query and the softmax weights P each go to the tensor cores as a high and
+// a low 16-bit part (x = hi + lo with hi = bf16(x), lo = bf16(x - hi), 16 significant bits together),
+// so q.k and P.V keep the precision that f16 operands give in one part.  With bf16's 8-bit
+// significand a single part moves q.k and the P weights by up to 2^-9 relative, more than the
+// decode tolerance allows; the low parts cost a second pass of each product on the tensor cores.
+template <int D, bool SPLIT_ = false>
 struct PfCfg {
+  static constexpr bool SPLIT = SPLIT_;
   static constexpr int SW = (2 * D) % 128 == 0 ? 128 : (2 * D) % 64 == 0 ? 64 : 32;
   static constexpr int SUB = SW / 2;  // columns per subtile
   static constexpr int NSUB = D / SUB;
@@ -56,11 +63,16 @@ struct PfCfg {
   // tile in TMEM and two K/V stages; larger heads run one CTA per SM with a double-buffered S tile.
   static constexpr int CPS = (D == 64 || D == 80) ? 2 : 1;  // CTAs per SM
   static constexpr int SBUF = CPS == 2 ? 1 : 2;              // S tiles in TMEM
-  static constexpr bool PSEP = D == 64;                      // P in TMEM columns of its own
+  static constexpr bool PSEP = D == 64 && !SPLIT;            // P in TMEM columns of its own
   static constexpr bool XQT = CPS == 2 && !PSEP;             // Q's mask column in TMEM, not smem
+  // SPLIT: the low part of the rotated query, the A operand of a second Q.K^T pass, lives in TMEM
+  // with two CTAs per SM (whose shared memory is full) and in shared memory with one
+  static constexpr bool QLO_TMEM = SPLIT && CPS == 2;
+  static constexpr bool QLO_SMEM = SPLIT && CPS == 1;
   static constexpr int NST = CPS == 2 ? 2 : D <= 96 ? 3 : 2;  // K/V stages
   static constexpr uint32_t Q_OFF = 0;
-  static constexpr uint32_t KV_OFF = TILE;
+  static constexpr uint32_t QLO_OFF = TILE;  // QLO_SMEM only
+  static constexpr uint32_t KV_OFF = TILE * (QLO_SMEM ? 2 : 1);
   // Mask columns: one 16-column subtile (32-byte swizzle) appended to Q (a constant) and to every K
   // stage (0 or a large negative number per key), so keys hidden from a whole query tile are masked
   // by the Q.K^T product itself.
@@ -78,12 +90,16 @@ struct PfCfg {
   // Q.K^T overlaps the softmax.  d_head 80 (two CTAs per SM): S [0,128) with P written over its
   // first 64 columns, O [128,208), Q's mask column [208,216) -- the next Q.K^T follows the P.V.
   // One CTA per SM: S0 [0,128), S1 [128,256), P written over the first 64 columns of its own S
-  // tile, then O0 and O1 (alternating per item).
+  // tile, then O0 and O1 (alternating per item).  SPLIT: P's high part over the first 64 columns of
+  // its S tile and its low part over the other 64 (d_head 64 then lays TMEM out as d_head 80 does);
+  // with two CTAs per SM the query's low part follows Q's mask column (D / 2 columns).
   static constexpr uint32_t P_COL = PSEP ? kPfRows : 0;  // else P lives in its S tile
+  static constexpr uint32_t PLO_COL = kPfRows / 2;       // SPLIT: P's low part, after its high part
   static constexpr int OBUF = SBUF == 1 ? 1 : 2;
   static constexpr uint32_t O_COL = SBUF == 2 ? 2 * kPfRows : PSEP ? kPfRows + kPfRows / 2 : kPfRows;
   static constexpr uint32_t XQ_COL = O_COL + OBUF * D;  // with XQT: 8 columns, 16 elements per row
-  static constexpr uint32_t TMEM_END = XQ_COL + (XQT ? 8 : 0);
+  static constexpr uint32_t QLO_COL = XQ_COL + (XQT ? 8 : 0);
+  static constexpr uint32_t TMEM_END = QLO_COL + (QLO_TMEM ? D / 2 : 0);
   static constexpr uint32_t TMEM_COLS = TMEM_END <= 256 ? 256 : 512;
   static_assert(TMEM_END <= TMEM_COLS && TMEM_COLS * CPS <= 512, "TMEM budget");
   static_assert(D % 16 == 0 && SW * NSUB == 2 * D, "bad tile geometry");
@@ -190,6 +206,10 @@ __device__ __forceinline__ void tmem_st8u(uint32_t taddr, const uint32_t* r) {
                "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
                : "memory");
 }
+__device__ __forceinline__ void tmem_st4u(uint32_t taddr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};" ::"r"(taddr), "r"(a), "r"(b), "r"(c), "r"(d)
+               : "memory");
+}
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ float ex2(float x) {
@@ -233,6 +253,24 @@ struct Pack16<BF16T> {
     return *reinterpret_cast<uint32_t*>(&h);
   }
 };
+
+// The two bf16 values of a packed pair as exact binary32 values (low half first).
+__device__ __forceinline__ float2 bf16x2_to_float2(uint32_t w) {
+  return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+}
+// SPLIT: x = hi + lo with hi, lo bf16 (a pair at a time): *hi = bf16(x) and the low part is the
+// bf16 rounding of x - hi, which binary32 holds exactly (x and hi agree in their leading bits).
+__device__ __forceinline__ uint32_t bf16_split2(float2 x, uint32_t* hi) {
+  *hi = Pack16<BF16T>::two(x.x, x.y);
+  const float2 h = bf16x2_to_float2(*hi);
+  const float2 d = __ffma2_rn(h, make_float2(-1.f, -1.f), x);
+  return Pack16<BF16T>::two(d.x, d.y);
+}
+
+template <typename T>
+constexpr bool kSplit = false;
+template <>
+constexpr bool kSplit<BF16T> = true;
 
 // 16-byte global -> shared copy that does not go through registers (src_bytes 0: zero fill).
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
@@ -323,7 +361,7 @@ template <typename T, int D>
 __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
     prefill_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_o, const PrefillArgs a) {
-  using Cf = PfCfg<D>;
+  using Cf = PfCfg<D, kSplit<T>>;
   constexpr int SW = Cf::SW, SUB = Cf::SUB, NST = Cf::NST, SBUF = Cf::SBUF;
   extern __shared__ uint8_t pf_smem_raw[];
   __shared__ uint64_t full_bar[NST], empty_bar[NST], s_full[SBUF], s_free;
@@ -497,6 +535,7 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
       constexpr uint32_t idS = mma_idesc(Pack16<T>::kType, 0, kPfRows, kPfRows);
       constexpr uint32_t idO = mma_idesc(Pack16<T>::kType, 1, kPfRows, D);
       const uint32_t q_s = smem_addr(sm + Cf::Q_OFF);
+      [[maybe_unused]] const uint32_t qlo_s = smem_addr(sm + Cf::QLO_OFF);
       const uint32_t xq_s = smem_addr(sm + Cf::XQ_OFF), xk_s = smem_addr(sm + Cf::XK_OFF);
       int64_t g = 0;
       bool ok = true;
@@ -526,6 +565,21 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
             tc_mma(tmem + sb * kPfRows, smem_desc(q_s + off, 16, 8 * SW, SW), smem_desc(k_s + off, 16, 8 * SW, SW),
                    idS, kk > 0);
           }
+          // SPLIT with RoPE: + Q_lo K^T (without RoPE the query is exact in the cache type)
+          if constexpr (Cf::SPLIT) {
+            if (a.rot > 0) {
+#pragma unroll
+              for (int kk = 0; kk < D / 16; ++kk) {
+                const uint32_t off = (kk * 16) / SUB * Cf::SUBB + (kk * 16) % SUB * 2;
+                if constexpr (Cf::QLO_TMEM)
+                  tc_mma_ts(tmem + sb * kPfRows, tmem + Cf::QLO_COL + 8 * kk, smem_desc(k_s + off, 16, 8 * SW, SW),
+                            idS, 1);
+                else
+                  tc_mma(tmem + sb * kPfRows, smem_desc(qlo_s + off, 16, 8 * SW, SW),
+                         smem_desc(k_s + off, 16, 8 * SW, SW), idS, 1);
+              }
+            }
+          }
           // + the mask column: 256 x (0 or -32768) per key
           if constexpr (Cf::XQT)
             tc_mma_ts(tmem + sb * kPfRows, tmem + Cf::XQ_COL, smem_desc(xk_s + st * kPfRows * 32, 16, 8 * 32, 32), idS, 1);
@@ -545,6 +599,11 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
 #pragma unroll
           for (int kk = 0; kk < kPfRows / 16; ++kk)
             tc_mma_ts(o_t, p_t + 8 * kk, smem_desc(v_s + kk * 16 * SW, Cf::SUBB, 8 * SW, SW), idO, (!first || kk > 0));
+          if constexpr (Cf::SPLIT) {  // + P_lo V
+#pragma unroll
+            for (int kk = 0; kk < kPfRows / 16; ++kk)
+              tc_mma_ts(o_t, p_t + Cf::PLO_COL + 8 * kk, smem_desc(v_s + kk * 16 * SW, Cf::SUBB, 8 * SW, SW), idO, 1);
+          }
           tc_commit(&pv_done);
           tc_commit(&empty_bar[st]);
           return true;
@@ -596,11 +655,53 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
       cp_async4(smem_addr(&qmeta[r]), a.meta + (valid ? w.ps.moff + iq : 0), valid ? 4u : 0u);
       cp_async_commit();
     };
+    // SPLIT: the address of chunk c8 of row r in the query's low-part tile (QLO_SMEM)
+    [[maybe_unused]] auto qlo_chunk = [&](int c8) -> uint32_t {
+      return q_chunk(c8) - smem_addr(sm + Cf::Q_OFF) + smem_addr(sm + Cf::QLO_OFF);
+    };
+    [[maybe_unused]] auto qlo_store = [&](int c8, uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3) {
+      if constexpr (Cf::QLO_TMEM)
+        tmem_st4u(tl + Cf::QLO_COL + 4 * c8, w0, w1, w2, w3);  // warp-collective: every lane stores
+      else
+        st_shared_v4(qlo_chunk(c8), w0, w1, w2, w3);
+    };
     auto q_finish = [&](const PfItem& w) {
       cp_async_wait_all();
       const int half = a.rot / 2;
       const int iq = w.qr0 + r;
-      if (half > 0 && iq < w.qr_end) {
+      if constexpr (Cf::SPLIT) {
+        // every row (rows past the tile's queries hold zeros), so the TMEM stores are warp-wide
+        if (half > 0) {
+          const int32_t qpos = iq < w.qr_end ? a.pos[a.off[w.s] + iq] : 0;
+          const int hc = half / 8;  // chunks per rotated half
+#pragma unroll
+          for (int c8 = 0; c8 < D / 16; ++c8) {
+            if (c8 < hc) {
+              const uint32_t a1 = q_chunk(c8), a2 = q_chunk(c8 + hc);
+              const uint4 u1 = ld_shared_v4(a1), u2 = ld_shared_v4(a2);
+              const uint32_t w1[4] = {u1.x, u1.y, u1.z, u1.w}, w2[4] = {u2.x, u2.y, u2.z, u2.w};
+              uint32_t h1[4], h2[4], l1[4], l2[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float2 x1 = T::f2(w1[e]), x2 = T::f2(w2[e]);
+                float sn0, cs0, sn1, cs1;
+                rope_sincos(qpos, a.rope_g[8 * c8 + 2 * e], &sn0, &cs0);
+                rope_sincos(qpos, a.rope_g[8 * c8 + 2 * e + 1], &sn1, &cs1);
+                l1[e] = bf16_split2(make_float2(x1.x * cs0 - x2.x * sn0, x1.y * cs1 - x2.y * sn1), &h1[e]);
+                l2[e] = bf16_split2(make_float2(x2.x * cs0 + x1.x * sn0, x2.y * cs1 + x1.y * sn1), &h2[e]);
+              }
+              st_shared_v4(a1, h1[0], h1[1], h1[2], h1[3]);
+              st_shared_v4(a2, h2[0], h2[1], h2[2], h2[3]);
+              qlo_store(c8, l1[0], l1[1], l1[2], l1[3]);
+              qlo_store(c8 + hc, l2[0], l2[1], l2[2], l2[3]);
+            }
+          }
+          // the dimensions past the rotary ones are exact: their low part is zero
+#pragma unroll
+          for (int c8 = 0; c8 < D / 8; ++c8)
+            if (c8 >= 2 * hc) qlo_store(c8, 0u, 0u, 0u, 0u);
+        }
+      } else if (half > 0 && iq < w.qr_end) {
         const int32_t qpos = a.pos[a.off[w.s] + iq];
         for (int c8 = 0; c8 < half / 8; ++c8) {
           const uint32_t a1 = q_chunk(c8), a2 = q_chunk(c8 + half / 8);
@@ -624,7 +725,7 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
       if constexpr (Cf::XQT) {
         const uint32_t wd[8] = {x01, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
         tmem_st8u(tl + Cf::XQ_COL, wd);
-        tmem_wait_st();
+        tmem_wait_st();  // also the query's low part (QLO_TMEM)
         tc_fence_before();
       } else {
         const uint32_t row = smem_addr(sm + Cf::XQ_OFF) + r * 32;
@@ -787,14 +888,21 @@ __global__ void __launch_bounds__(kPfThreads, PfCfg<D>::CPS)
 #pragma unroll
         for (int q = 0; q < CW / 32; ++q) {
           uint32_t pk[16];
+          [[maybe_unused]] uint32_t pl[16];
 #pragma unroll
           for (int c = 0; c < 32; c += 2) {
             const float2 x = __ffma2_rn(make_float2(sv[32 * q + c], sv[32 * q + c + 1]), c2v, nref);
             const float2 p = make_float2(ex2(x.x), ex2(x.y));
             rs4[(c >> 1) & 3] = __fadd2_rn(rs4[(c >> 1) & 3], p);
-            pk[c / 2] = Pack16<T>::two(p.x, p.y);
+            if constexpr (Cf::SPLIT)
+              pl[c / 2] = bf16_split2(p, &pk[c / 2]);
+            else
+              pk[c / 2] = Pack16<T>::two(p.x, p.y);
           }
           if (sok) tmem_st16u(p_tl + 16 * q, pk);
+          if constexpr (Cf::SPLIT) {
+            if (sok) tmem_st16u(p_tl + Cf::PLO_COL + 16 * q, pl);
+          }
         }
         const float rs = ((rs4[0].x + rs4[0].y) + (rs4[1].x + rs4[1].y)) + ((rs4[2].x + rs4[2].y) + (rs4[3].x + rs4[3].y));
         l = l * alpha + rs;
@@ -946,6 +1054,7 @@ cudaError_t encode_plane(const Geometry& g, void* base, unsigned char* out) {
 
 template <typename T, int D>
 cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int64_t grid, cudaStream_t stream) {
+  using Cf = PfCfg<D, kSplit<T>>;
   static std::mutex mu;
   static bool attr_set[64] = {};  // per device: the shared-memory opt-in and the register check
   int dev = 0;
@@ -957,15 +1066,15 @@ cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int6
   std::lock_guard<std::mutex> lock(mu);
   if (!attr_set[dev]) {
     const cudaError_t e = cudaFuncSetAttribute(prefill_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)PfCfg<D>::SMEM);
+                                               (int)Cf::SMEM);
     if (e != cudaSuccess) return e;
-    if (PfCfg<D>::CPS == 2) {
+    if (Cf::CPS == 2) {
       // the setmaxnreg shares assume each thread starts with exactly REG_LAUNCH registers; with
       // fewer the softmax warpgroup's increase could never be granted, so refuse to launch
       cudaFuncAttributes fa;
       const cudaError_t e2 = cudaFuncGetAttributes(&fa, prefill_kernel<T, D>);
       if (e2 != cudaSuccess) return e2;
-      if (fa.numRegs != PfCfg<D>::REG_LAUNCH) return cudaErrorInvalidConfiguration;
+      if (fa.numRegs != Cf::REG_LAUNCH) return cudaErrorInvalidConfiguration;
     }
     attr_set[dev] = true;
   }
@@ -973,7 +1082,7 @@ cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int6
   std::memcpy(&mk, maps.k, sizeof mk);
   std::memcpy(&mv, maps.v, sizeof mv);
   std::memset(&mo, 0, sizeof mo);
-  if (PfCfg<D>::OSTAGE && a.n_qtok >= kPfRows) {
+  if (Cf::OSTAGE && a.n_qtok >= kPfRows) {
     // out as [token][head][D] fp32, stored in boxes of 32 columns x one head x 32 tokens from the
     // softmax warps' swizzled staging buffers (only full query tiles take this path)
     cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.H, (cuuint64_t)a.n_qtok};
@@ -985,7 +1094,7 @@ cudaError_t launch_prefill_t(const PrefillMaps& maps, const PrefillArgs& a, int6
                                 CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
   }
-  prefill_kernel<T, D><<<(unsigned)grid, kPfThreads, PfCfg<D>::SMEM, stream>>>(mk, mv, mo, a);
+  prefill_kernel<T, D><<<(unsigned)grid, kPfThreads, Cf::SMEM, stream>>>(mk, mv, mo, a);
   return cudaGetLastError();
 }
 

@@ -21,10 +21,10 @@ from _parity import MAX_ABS, MAX_REL, REL_FLOOR, check_metadata
 
 pytestmark = pytest.mark.gpu
 
-# The kernel rounds the rotated query and the softmax weights P to the cache type for the 16-bit
-# tensor-core products (q.k and P.V, fp32 accumulation).  With f16 (unit roundoff 2^-11) that stays
-# inside the decode tolerance; bf16 has 8x the unit roundoff (2^-8), and its bound is scaled by 8.
-TOL = {"f16": (MAX_ABS, MAX_REL), "bf16": (8 * MAX_ABS, 8 * MAX_REL)}
+# One tolerance for both 16-bit types, the decode's (fp16/bf16 K/V with fp32 accumulation).  The
+# kernel feeds the rotated query and the softmax weights P to the tensor cores in the cache type; with
+# bf16 it passes each as a high and a low bf16 part, so both products keep 16 significant bits.
+TOL = {"f16": (MAX_ABS, MAX_REL), "bf16": (MAX_ABS, MAX_REL)}
 
 
 def _compare(got, ref, dtype, what):
@@ -173,10 +173,14 @@ def test_prefill_blocks_of_512_cl_key_in_last_column():
     run_prefill(w, 512, layers=[0], heads=[0, 31])
 
 
-def test_prefill_rope_bf16():
-    # the query rotation rounded to bf16 (held to eight times the f16 bound)
-    w = dataclasses.replace(wl.rope3b(32, b=2, L=400, M=1), dtype="bf16", name="rope-bf16")
-    run_prefill(w, 0, layers=[0], heads=[0, 31])
+@pytest.mark.parametrize("d,rot,block", [(80, 80, 0), (80, 32, 200), (64, 64, 0), (96, 96, 0), (128, 64, 256)])
+def test_prefill_rope_bf16(d, rot, block):
+    # bf16 with RoPE: the rotated query goes to the tensor cores as a high and a low bf16 part (its low
+    # part in TMEM with two CTAs per SM, d_head 64 / 80, and in shared memory with one, d_head 96 /
+    # 128; zero past the rotary dimensions), P likewise; held to the f16 bound
+    w = dataclasses.replace(wl.rope3b(32, b=2, L=400, M=1), dtype="bf16", d=d, rotary_dim=rot,
+                            scale=1.0 / math.sqrt(d), name=f"rope-bf16-d{d}-r{rot}")
+    run_prefill(w, block, layers=[0], heads=[0, 31])
 
 
 @pytest.mark.parametrize("d,rot", [(96, 96), (128, 64)])
