@@ -218,6 +218,19 @@ class Runner:
                 self.open_cl[s] = -1
         return seq, cl, cr
 
+    def append_only(self, inp: StepInputs, stream=None):
+        """The first part of a step: append the token's K/V rows of every layer (decode follows)."""
+        self.cache.append(inp.kv_k, inp.kv_v, np.ones(self.w.b, dtype=np.int32), inp.kinds, layer=-1,
+                          stream=kvc.stream_handle(stream))
+
+    def finish_step(self, inp: StepInputs, stream=None):
+        """The last part of a step after its decode: free the span the token closed, if any."""
+        seq, cl, cr = self.step_spans(inp.kinds)
+        self.g += 1
+        if seq:
+            self.cache.compress_spans(seq, cl, cr, kvc.stream_handle(stream))
+        return seq
+
     def step(self, inp: StepInputs, out: torch.Tensor, stream=None, events=None, compress: bool = True):
         """One decode step: append the token, decode all M layers into out[M][b][H][d], free closed spans.
 

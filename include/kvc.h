@@ -195,8 +195,8 @@ const kvc_book* kvc_get_book(const kvc_cache* cache);
 kvc_status kvc_append(kvc_cache* cache, int layer, const void* k, const void* v, const int32_t* n_new,
                       const int32_t* pos, const uint8_t* kinds, void* stream);
 
-/* kvc_append with write-time freeing (Sec. 3.1: the enclosed KV is freed "in one go" after a
- * prefix, or block by block for long prefixes): spans that both open and close among the new
+/* kvc_append with write-time freeing (Sec. 3.1: the enclosed KV can be released all at once after
+ * a prefix, or block by block for long prefixes): spans that both open and close among the new
  * tokens of a sequence are freed as the tokens are written -- their <CL> (paper policy) and
  * enclosed rows are never stored, so no compaction has to move anything for them.  Spans closed
  * here but opened by an earlier call, or still open, are stored as by kvc_append (free the former
@@ -227,8 +227,11 @@ kvc_status kvc_decode_attention(kvc_cache* cache, int layer, const void* q, floa
  * model whose queries for all those layers are ready, as in the paper's throughput setting,
  * Sec. 4.3): layer first + i reads q + i * q_layer_stride elements of the cache dtype and writes
  * out + i * out_layer_stride floats; strides are in elements, each layer's slice laid out as for
- * kvc_decode_attention.  The same launches as n_layers separate calls, in layer order on `stream`;
- * on an error the layers before the failing one have been launched. */
+ * kvc_decode_attention.  When every (sequence, head) segment holds about as many rows as the others
+ * (the longest at most 1.3x the mean), one launch covers every layer's segments, each processed
+ * whole by one warp exactly as a per-layer launch with the same tile shape does it; otherwise the
+ * layers are launched one by one, in order, on `stream`, and on an error the layers before the
+ * failing one have been launched. */
 kvc_status kvc_decode_attention_layers(kvc_cache* cache, int first, int n_layers, const void* q, int64_t q_layer_stride,
                                        float scale, float* out, int64_t out_layer_stride, void* stream);
 
@@ -262,7 +265,7 @@ kvc_status kvc_decode_attention_static_scratch(kvc_cache* cache, int layer, cons
  *   scale: > 0.
  * The queries' own K/V rows must be stored: append a block with kvc_append (every layer up to
  * `layer` written), run the prefill of each layer, then free the spans the block closed with
- * kvc_compress_spans -- the "for-loop over blocks" of Sec. 3.1.  Spans closed earlier may still be
+ * kvc_compress_spans -- the block-by-block loop of Sec. 3.1.  Spans closed earlier may still be
  * stored (their rows are masked), so a whole prompt can also be appended and run in one call.
  * Errors: KVC_ERR_STATE when a query token is not stored (for example freed by
  * kvc_append_free_closed) or its layer is not written; KVC_ERR_UNSUPPORTED under
@@ -290,6 +293,18 @@ kvc_status kvc_check_bounded_wait(kvc_cache* cache, uint64_t limit_ns, void* str
 
 /* Number of kernels this cache has launched so far. */
 int64_t kvc_launch_count(const kvc_cache* cache);
+
+/* Measurement of the two compaction kernels (Sec. 3.1, freeing the enclosed KV): with enable != 0,
+ * every later kvc_compress_spans that moves rows records CUDA events on its stream before the keep
+ * flag scan, between the scan and the row moves, and after the row moves (0 turns this off).  The
+ * event between the kernels keeps the row moves from being scheduled before the scan completes, so
+ * a timed compaction can take a few microseconds longer than an untimed one.  The events are created
+ * on the current device at the first timed call and freed by kvc_destroy. */
+kvc_status kvc_set_compaction_timing(kvc_cache* cache, int enable);
+
+/* Durations in milliseconds of the last compaction's scan and row moves (synchronous: waits for
+ * its last event).  KVC_ERR_STATE if the last kvc_compress_spans was not timed or moved nothing. */
+kvc_status kvc_last_compaction_ms(kvc_cache* cache, float* scan_ms, float* move_ms);
 
 /* How the last decode launch divided its work (host-side record, no synchronisation):
  * plan[0] = mode (0: the kept rows split evenly over a full wave of warps, split (sequence, head)

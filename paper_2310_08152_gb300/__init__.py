@@ -332,6 +332,18 @@ def kvc_launch_count(cache: int) -> int:
     return lib().kvc_launch_count(cache)
 
 
+def kvc_set_compaction_timing(cache: int, enable: bool):
+    _check(lib().kvc_set_compaction_timing(cache, 1 if enable else 0))
+
+
+def kvc_last_compaction_ms(cache: int):
+    """(scan ms, row-move ms) of the last timed compaction."""
+    a = ctypes.c_float()
+    b = ctypes.c_float()
+    _check(lib().kvc_last_compaction_ms(cache, ctypes.byref(a), ctypes.byref(b)))
+    return float(a.value), float(b.value)
+
+
 def kvc_last_decode_plan(cache: int) -> dict:
     a = np.zeros(4, np.int32)
     _check(lib().kvc_last_decode_plan(cache, a.ctypes.data))

@@ -64,6 +64,8 @@ SIGNATURES = [
     ("kvc_launch_count", c_int64, [P]),
     ("kvc_check_bounded_wait", c_int, [P, ctypes.c_uint64, P]),
     ("kvc_last_decode_plan", c_int, [P, P]),
+    ("kvc_set_compaction_timing", c_int, [P, c_int]),
+    ("kvc_last_compaction_ms", c_int, [P, P, P]),
 ]
 
 _lib = None

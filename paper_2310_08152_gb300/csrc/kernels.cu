@@ -494,12 +494,16 @@ struct DecodeCfg {
 };
 
 struct DecodeDev {
-  const uint16_t* k;  // layer plane
+  const uint16_t* k;  // plane of the launch's first layer
   const uint16_t* v;
   const DState* ds;
   const int64_t* P;
-  int64_t R;
+  int64_t R;          // rows of one layer (H * P[b])
   int NW;  // workers (warps)
+  int n_layers;       // layers of this launch; layer i's segments follow layer i-1's
+  int64_t plane;      // elements between consecutive layers' K (or V) planes
+  int64_t q_stride;   // elements between consecutive layers' queries
+  int64_t out_stride; // floats between consecutive layers' outputs
   const uint16_t* q;
   float* out;
   float* partials;
@@ -511,11 +515,11 @@ struct DecodeDev {
   int seg_per_worker;  // k > 0: worker w owns segments [w k, w k + k) whole; 0: stream-K split of the rows
 };
 
-// The tiles of a worker: its flat row range [x, hi) of the concatenation over (sequence, head)
-// segments, cut into tiles of at most TR rows that never cross a segment.
+// The tiles of a worker: its flat row range [x, hi) of the concatenation over (layer, sequence,
+// head) segments, cut into tiles of at most TR rows that never cross a segment.
 struct TileIter {
   int64_t x, hi, Lc, r;
-  int s, h;
+  int s, h, layer;
   __device__ __forceinline__ bool done() const { return x >= hi; }
   // rows of the next tile: at most TR, never past the segment, the range, or a ring's end (wrap)
   __device__ __forceinline__ int n(int TR, int64_t wrap) const {
@@ -524,7 +528,8 @@ struct TileIter {
     if (r < wrap && wrap - r < k) k = wrap - r;
     return (int)(k < TR ? k : TR);
   }
-  __device__ __forceinline__ void advance(int n, const int64_t* P, int H) {
+  // x < hi guarantees a later segment with rows, in this layer or a later one of the launch
+  __device__ __forceinline__ void advance(int n, const int64_t* P, int H, int b) {
     x += n;
     r += n;
     if (r == Lc && x < hi) {
@@ -532,7 +537,10 @@ struct TileIter {
       if (++h == H) {
         h = 0;
         do {
-          ++s;
+          if (++s == b) {
+            s = 0;
+            ++layer;
+          }
         } while (P[s + 1] == P[s]);
         Lc = P[s + 1] - P[s];
       }
@@ -541,6 +549,23 @@ struct TileIter {
 };
 
 __device__ __forceinline__ int worker_of(int64_t x, int64_t R, int NW) { return (int)(((x + 1) * NW - 1) / R); }
+
+// The sequence holding flat row o of a layer (0 <= o < H P[b]): the largest s < b with H P[s] <= o,
+// which is a sequence with rows.  A 32-ary search by the whole warp: each round probes 32 evenly
+// spaced candidates with one load per lane and keeps the interval after the last one that holds.
+__device__ __forceinline__ int seq_of_row(const int64_t* P, int b, int H, int64_t o, int lane) {
+  int a = 0, z = b;  // the answer lies in [a, z)
+  while (z - a > 1) {
+    const int step = (z - a + 31) / 32;
+    const int k = a + lane * step;
+    const bool le = k < z && (int64_t)H * P[k] <= o;
+    const unsigned bal = __ballot_sync(0xFFFFFFFFu, le);
+    const int j = 31 - __clz(bal);  // bal != 0: candidate a always holds
+    a = a + j * step;
+    z = min(z, a + step);
+  }
+  return a;
+}
 
 
 
@@ -561,19 +586,24 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
     return;
   }
   const int H = g.H;
+  const int64_t segs_layer = (int64_t)g.b * H;
   int64_t lo, hi;
-  int s_first = 0;
-  if (p.seg_per_worker) {  // segments [sg0, sg1] = (s, h) pairs in order, each whole
+  if (p.seg_per_worker) {  // segments [sg0, sg1) = (layer, s, h) triples in order, each whole
+    // first flat row of segment sg (sg = n_layers * b * H gives the end of the last layer)
+    auto seg_row = [&](int64_t sg) {
+      const int64_t l = sg / segs_layer, w = sg - l * segs_layer;
+      const int s = (int)(w / H);
+      const int64_t a = p.P[s], z = p.P[s + 1];
+      return l * p.R + (int64_t)H * a + (w - (int64_t)s * H) * (z - a);
+    };
     const int64_t sg0 = (int64_t)wid * p.seg_per_worker;
-    const int64_t sg1 = min(sg0 + p.seg_per_worker, (int64_t)g.b * H) - 1;
-    s_first = (int)(sg0 / H);
-    const int s1 = (int)(sg1 / H);
-    const int64_t a0 = p.P[s_first], z0 = p.P[s_first + 1], a1 = p.P[s1], z1 = p.P[s1 + 1];
-    lo = (int64_t)H * a0 + (sg0 - (int64_t)s_first * H) * (z0 - a0);
-    hi = (int64_t)H * a1 + (sg1 - (int64_t)s1 * H + 1) * (z1 - a1);
+    const int64_t sg1 = min(sg0 + p.seg_per_worker, (int64_t)p.n_layers * segs_layer);
+    lo = seg_row(sg0);
+    hi = seg_row(sg1);
   } else {
-    lo = (int64_t)wid * p.R / p.NW;
-    hi = (int64_t)(wid + 1) * p.R / p.NW;
+    const int64_t Rt = (int64_t)p.n_layers * p.R;
+    lo = (int64_t)wid * Rt / p.NW;
+    hi = (int64_t)(wid + 1) * Rt / p.NW;
   }
   if (lo >= hi) {
     pdl_wait();
@@ -595,19 +625,11 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   fence_proxy_async_smem();
   __syncwarp();
 
-  // segment holding row `lo`: s = (number of sequences with H*P[s] <= lo) - 1
-  int cnt = 0;
-  if (p.seg_per_worker) {
-    cnt = s_first + 1;
-  } else {
-    for (int base_s = 0; base_s < g.b; base_s += 32) {
-      const int k = base_s + lane;
-      const bool le = k < g.b && (int64_t)H * p.P[k] <= lo;
-      cnt += __popc(__ballot_sync(kFull, le));
-    }
-  }
+  // the segment holding row `lo`: its layer, then the sequence with rows that holds the offset
   TileIter ci;  // consumed tiles
-  ci.s = cnt - 1;
+  ci.layer = (int)(lo / p.R);
+  const int64_t o_layer = lo - (int64_t)ci.layer * p.R;
+  ci.s = seq_of_row(p.P, g.b, H, o_layer, lane);
   // everything that depends only on the starting sequence, loaded together
   const int64_t P0 = p.P[ci.s], P1 = p.P[ci.s + 1];
   const DState ds0 = p.ds[ci.s];
@@ -616,7 +638,7 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   int seg_cap = st.cap[ci.s];
   ci.Lc = P1 - P0;
   {
-    const int64_t o = lo - (int64_t)H * P0;
+    const int64_t o = o_layer - (int64_t)H * P0;
     ci.h = (int)(o / ci.Lc);
     ci.r = o - (int64_t)ci.h * ci.Lc;
   }
@@ -639,9 +661,10 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
     const int64_t row = seg_row0 + (int64_t)ii.h * seg_cap + slot;
     const uint32_t bytes = (uint32_t)n * L::RB;
     mbar_arrive_expect_tx(&full[stage], 2 * bytes);
-    bulk_g2s(stg + stage * 2 * C::TILE, p.k + row * D, bytes, &full[stage]);
-    bulk_g2s(stg + stage * 2 * C::TILE + C::TILE, p.v + row * D, bytes, &full[stage]);
-    ii.advance(n, p.P, H);
+    const int64_t e0 = (int64_t)ii.layer * p.plane + row * D;
+    bulk_g2s(stg + stage * 2 * C::TILE, p.k + e0, bytes, &full[stage]);
+    bulk_g2s(stg + stage * 2 * C::TILE + C::TILE, p.v + e0, bytes, &full[stage]);
+    ii.advance(n, p.P, H, g.b);
   };
   int issued = 0;
   // K/V of this layer are not written by the preceding decode: stream them before it completes
@@ -662,8 +685,8 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   // raw q of the next piece (and its rotation partner), fetched one tile ahead of its use
   constexpr int QPL = (D + 31) / 32;
   float qa[QPL], qb[QPL];
-  auto fetch_q = [&](int s_, int h_) {
-    const uint16_t* qrow = p.q + ((int64_t)s_ * H + h_) * D;
+  auto fetch_q = [&](int l_, int s_, int h_) {
+    const uint16_t* qrow = p.q + (int64_t)l_ * p.q_stride + ((int64_t)s_ * H + h_) * D;
     const int half = g.rot / 2;
 #pragma unroll
     for (int j = 0; j < QPL; ++j) {
@@ -676,7 +699,7 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
       }
     }
   };
-  fetch_q(ci.s, ci.h);
+  fetch_q(ci.layer, ci.s, ci.h);
   DState dn = ds0;
   const int grp = lane / L::LPR;
   const int tl = lane % L::LPR;
@@ -691,7 +714,7 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   int t = 0;     // tiles consumed
   int t_ok = 0;  // tiles whose copies were seen complete
   while (!ci.done()) {
-    const int s = ci.s, h = ci.h;
+    const int s = ci.s, h = ci.h, layer = ci.layer;
     const int64_t r0 = ci.r;
     if (piece_start && s != cur_s) {  // the next sequence's state was prefetched with its q
       cur_s = s;
@@ -740,8 +763,8 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
     }
     if (r0 + n == ci.Lc && ci.x + n < ci.hi) {  // this tile ends the segment: fetch the next piece's q
       TileIter nx = ci;
-      nx.advance(n, p.P, H);
-      fetch_q(nx.s, nx.h);
+      nx.advance(n, p.P, H, g.b);
+      fetch_q(nx.layer, nx.s, nx.h);
       if (nx.s != s) dn = p.ds[nx.s];
     }
     if (!dead) {
@@ -811,7 +834,7 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
     }
     __syncwarp();
     const bool seg_done = (r0 + n == ci.Lc);
-    ci.advance(n, p.P, H);
+    ci.advance(n, p.P, H, g.b);
     ++t;
     bool refilled = false;
     if (seg_done || ci.done()) {
@@ -842,12 +865,16 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
       if (!dead) {
         if (piece_whole && seg_done) {
           const float inv = 1.f / Ls;
+          float* orow = p.out + (int64_t)layer * p.out_stride + (int64_t)seg * D;
           for (int col = lane; col < D; col += 32) {
             float O = 0.f;
 #pragma unroll
             for (int r = 0; r < L::RPI; ++r) O += red[r * D + col];
-            p.out[(int64_t)seg * D + col] = O * inv;
+            orow[col] = O * inv;
           }
+        } else if (p.n_layers > 1) {
+          // launches over several layers take whole segments only (the host plans no split)
+          if (lane == 0) atomicOr(p.status, STATUS_CHECK);
         } else {
           float* pp = p.partials + (int64_t)(wid + seg) * (D + 4);
           for (int col = lane; col < D; col += 32) {
@@ -962,6 +989,10 @@ cudaError_t launch_decode_cfg(const Geometry& g, const Static& st, const Buffers
   p.P = a.P;
   p.R = a.R;
   p.NW = (int)NW;
+  p.n_layers = a.n_layers < 1 ? 1 : a.n_layers;
+  p.plane = plane;
+  p.q_stride = a.q_layer_stride;
+  p.out_stride = a.out_layer_stride;
   p.q = static_cast<const uint16_t*>(a.q);
   p.out = a.out;
   p.partials = a.partials;
@@ -998,6 +1029,11 @@ inline SegSplit seg_split(int64_t nseg, int occ, int num_sms) {
   return {k, workers, (workers + num_sms - 1) / num_sms * k};
 }
 
+// Segments of the uploaded state are balanced: the longest holds at most 1.3x the mean rows.
+inline bool decode_balanced(const DecodeArgs& a) {
+  return a.n_segments > 0 && 10 * a.max_segment * a.n_segments <= 13 * a.R;
+}
+
 template <typename T, int D>
 cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a, int num_sms,
                             cudaStream_t stream, int* grid, DecodePlan* plan) {
@@ -1005,14 +1041,16 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   constexpr int BK = KVC_DEC_SEG2_KPT, BS = KVC_DEC_SEG2_STAGES;
   constexpr int TK = KVC_DEC_STREAM_KPT, TS = KVC_DEC_STREAM_STAGES;
   // Balanced segments (longest within 1.3x of the mean) are never split, so no warp writes split-K
-  // partials or waits on a combine: one warp per (sequence, head) segment when a wave of resident
-  // warps holds them all (the wider pipeline shape first), else k consecutive whole segments per
-  // warp, with the shape and k that put the fewest segments on the busiest SM.  Otherwise the
-  // rows are split evenly over a full wave (stream-K).
-  const int64_t nseg = (int64_t)g.b * g.H;
-  const bool balanced = a.n_segments > 0 && nseg <= kMaxDecodeWorkers && 10 * a.max_segment * a.n_segments <= 13 * a.R;
-  cudaError_t e;
-  if (balanced) {
+  // partials or waits on a combine: one warp per (layer, sequence, head) segment when a wave of
+  // resident warps holds them all (the wider pipeline shape first), else k consecutive whole
+  // segments per warp, with the shape and k that put the fewest segments on the busiest SM.
+  // Otherwise the rows are split evenly over a full wave (stream-K), one layer per launch.
+  const int n_layers = a.n_layers < 1 ? 1 : a.n_layers;
+  const int64_t nseg = (int64_t)n_layers * g.b * g.H;
+  if (!decode_balanced(a)) {
+    if (n_layers > 1) return cudaErrorNotSupported;  // the caller launches the layers one by one
+  } else {
+    cudaError_t e;
     int occ_a = 0, occ_b = 0;
     e = decode_occupancy<T, D, AK, AS>(&occ_a);
     if (e == cudaSuccess) e = decode_occupancy<T, D, BK, BS>(&occ_b);
@@ -1033,6 +1071,7 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
     *plan = {3, (int)sb.workers, BK * Lanes<D>::RPI, BS};
     return launch_decode_cfg<T, D, BK, BS>(g, st, buf, a, sb.workers, sb.k, stream, grid);
   }
+  cudaError_t e;
   int occ = 0;
   e = decode_occupancy<T, D, TK, TS>(&occ);
   if (e != cudaSuccess) return e;
@@ -1106,7 +1145,8 @@ cudaError_t launch_append(const Geometry& g, const Static& st, const Buffers& bu
 }
 
 cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& buf, const AffSeq* aff, int n_aff,
-                           const int32_t* ranges, int32_t* src_map, cudaStream_t stream, int* launched) {
+                           const int32_t* ranges, int32_t* src_map, cudaStream_t stream, int* launched,
+                           cudaEvent_t between) {
   *launched = 0;
   if (n_aff <= 0) return cudaSuccess;
   compact_scan_kernel<<<n_aff, kScanThreads, 0, stream>>>(st, buf, aff, reinterpret_cast<const int2*>(ranges),
@@ -1114,6 +1154,10 @@ cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& b
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   *launched = 1;
+  if (between != nullptr) {
+    e = cudaEventRecord(between, stream);
+    if (e != cudaSuccess) return e;
+  }
   const int64_t blocks = (int64_t)n_aff * g.M * 2 * g.H;
   e = by_dhead(g.D, [&](auto dc) {
     constexpr int D = decltype(dc)::value;

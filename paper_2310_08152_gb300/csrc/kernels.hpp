@@ -73,16 +73,21 @@ inline size_t append_maps_bytes(int b) { return 2 * 128 * (size_t)b; }
 cudaError_t encode_append_maps(const Geometry& g, const Buffers& buf, const int64_t* seq_row0, const int32_t* cap,
                                unsigned char* out);
 
+// Scan, then row moves.  between: an event recorded on the stream between the two kernels, or NULL.
 cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& buf, const AffSeq* aff, int n_aff,
-                           const int32_t* ranges, int32_t* src_map, cudaStream_t stream, int* launched);
+                           const int32_t* ranges, int32_t* src_map, cudaStream_t stream, int* launched,
+                           cudaEvent_t between = nullptr);
 
 struct DecodeArgs {
-  int layer;
+  int layer;             // the first layer of the launch
+  int n_layers = 1;      // layers layer .. layer + n_layers - 1 in one launch (balanced segments only)
   const DState* dstate;  // [b]
   const int64_t* P;      // [b+1] prefix sums of attended-range lengths (len - begin)
   int64_t R;             // H * P[b]
-  const void* q;         // [b][H][D]
-  float* out;            // [b][H][D]
+  const void* q;         // [b][H][D] per layer, layer i at q + i * q_layer_stride elements
+  float* out;            // [b][H][D] per layer, layer i at out + i * out_layer_stride floats
+  int64_t q_layer_stride = 0;
+  int64_t out_layer_stride = 0;
   float scale;
   float* partials;       // [(kMaxDecodeWorkers + b*H) * (D + 4)]
   int* counters;         // [b*H], zero between launches
@@ -96,12 +101,15 @@ struct DecodeArgs {
 };
 
 // How a decode launch split its work: mode 0 = stream-K over all rows, 1 / 2 = one warp per
-// (sequence, head) segment with the wide / narrow pipeline; workers = warps; tile rows; stages.
+// (layer, sequence, head) segment with the wide / narrow pipeline, 3 = several consecutive whole
+// segments per warp; workers = warps; tile rows; stages.
 struct DecodePlan {
   int mode, workers, tile_rows, stages;
 };
 
-// Returns the grid used through *grid (0 if nothing launched) and the plan through *plan.
+// Returns the grid used through *grid (0 if nothing launched) and the plan through *plan.  A launch
+// over several layers (a.n_layers > 1) takes whole segments only: when the segments are not
+// balanced it launches nothing and returns cudaErrorNotSupported, and the caller goes layer by layer.
 cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a,
                           int num_sms, cudaStream_t stream, int* grid, DecodePlan* plan);
 

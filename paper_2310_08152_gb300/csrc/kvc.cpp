@@ -238,6 +238,10 @@ struct kvc_cache {
   int pre_ctas = 0;
   kvc::PrefillMaps maps;
   bool amaps_ok = false;  // the append kernel's TMA descriptors are in the workspace
+  // compaction timing (kvc_set_compaction_timing): events before the scan, between the kernels, after
+  bool time_compaction = false;
+  bool timed_compaction = false;  // the last compaction recorded them
+  cudaEvent_t cev[3] = {nullptr, nullptr, nullptr};
 
   kvc_cache(const kvc_config& c, int64_t C_)
       : cfg(c), C(C_), bk(c.b, (kvc::Policy)c.policy, c.seq_capacity, (double)c.local_ratio) {
@@ -250,6 +254,11 @@ struct kvc_cache {
     }
     ws = ws_layout(c.b, c.H, c.d_head, c.rotary_dim, C);
     layers_done = c.M;
+  }
+
+  ~kvc_cache() {
+    for (auto& e : cev)
+      if (e) cudaEventDestroy(e);
   }
 
   unsigned char* wsp(size_t o) const { return static_cast<unsigned char*>(cfg.workspace) + o; }
@@ -761,28 +770,44 @@ kvc_status kvc_compress_spans(kvc_cache* c, const int32_t* seq, const int64_t* c
   e = c->ring.commit(c->wsp(c->ws.dyn), bytes, stream);
   if (e != cudaSuccess) return cuda_fail(e, "upload compaction plan");
   int launched = 0;
+  const bool timed = c->time_compaction && n_aff > 0;
+  c->timed_compaction = false;
+  if (timed) {
+    for (auto& ev : c->cev)
+      if (!ev && (e = cudaEventCreate(&ev)) != cudaSuccess) return cuda_fail(e, "cudaEventCreate");
+    if ((e = cudaEventRecord(c->cev[0], stream)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+  }
   e = kvc::launch_compact(c->geom(), c->stat(), c->bufs(),
                           reinterpret_cast<const kvc::AffSeq*>(c->wsp(c->ws.dyn + c->ws.dyn_payload)), n_aff,
                           reinterpret_cast<const int32_t*>(c->wsp(c->ws.dyn + c->ws.dyn_payload + aff_bytes)),
-                          reinterpret_cast<int32_t*>(c->wsp(c->ws.src_map)), stream, &launched);
+                          reinterpret_cast<int32_t*>(c->wsp(c->ws.src_map)), stream, &launched,
+                          timed ? c->cev[1] : nullptr);
   c->launches += launched;
   c->last_was_decode = false;
   if (e != cudaSuccess) return cuda_fail(e, "compaction kernels");
+  if (timed) {
+    if ((e = cudaEventRecord(c->cev[2], stream)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    c->timed_compaction = true;
+  }
   return ok();
 }
 
-kvc_status kvc_decode_attention(kvc_cache* c, int layer, const void* q, float scale, float* out, void* stream_) {
+// Checks shared by the decode entry points, for layers [layer, layer + n_layers).
+static kvc_status decode_check(kvc_cache* c, int layer, int n_layers, const void* q, float scale, float* out) {
   if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
-  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
-  if (layer < 0 || layer >= c->cfg.M) return fail(KVC_ERR_INVALID_ARG, "layer %d out of range", layer);
+  if (n_layers < 1 || layer < 0 || layer + n_layers > c->cfg.M)
+    return fail(KVC_ERR_INVALID_ARG, "layers [%d, %d) out of range [0, %d)", layer, layer + n_layers, c->cfg.M);
   if (!q || !out) return fail(KVC_ERR_INVALID_ARG, "q/out are NULL");
   if (!std::isfinite(scale)) return fail(KVC_ERR_INVALID_ARG, "scale is not finite");
-  if (layer >= c->layers_done) return fail(KVC_ERR_STATE, "layer %d of the last tokens is not written yet", layer);
+  if (layer + n_layers > c->layers_done)
+    return fail(KVC_ERR_STATE, "layer %d of the last tokens is not written yet", std::max(layer, c->layers_done));
   if (!c->cuda_ready) return fail(KVC_ERR_STATE, "nothing appended yet");
   if (!c->decode_ok) return fail(KVC_ERR_STATE, "%s", c->decode_err.c_str());
   if (c->R <= 0) return fail(KVC_ERR_STATE, "no sequence has a token to query");
-  kvc_status st = c->ensure_cuda(stream);
-  if (st != KVC_OK) return st;
+  return KVC_OK;
+}
+
+static kvc::DecodeArgs decode_args(kvc_cache* c, int layer, const void* q, float scale, float* out) {
   kvc::DecodeArgs a;
   a.layer = layer;
   a.dstate = reinterpret_cast<const kvc::DState*>(c->wsp(c->ws.dyn));
@@ -797,6 +822,16 @@ kvc_status kvc_decode_attention(kvc_cache* c, int layer, const void* q, float sc
   a.kv_before_wait = c->last_was_decode ? 1 : 0;
   a.n_segments = c->n_segments;
   a.max_segment = c->max_segment;
+  return a;
+}
+
+kvc_status kvc_decode_attention(kvc_cache* c, int layer, const void* q, float scale, float* out, void* stream_) {
+  kvc_status st = decode_check(c, layer, 1, q, scale, out);
+  if (st != KVC_OK) return st;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  st = c->ensure_cuda(stream);
+  if (st != KVC_OK) return st;
+  const kvc::DecodeArgs a = decode_args(c, layer, q, scale, out);
   int grid = 0;
   cudaError_t e = kvc::launch_decode(c->geom(), c->stat(), c->bufs(), a, c->num_sms, stream, &grid, &c->last_plan);
   if (e != cudaSuccess) return cuda_fail(e, "decode kernel");
@@ -806,18 +841,41 @@ kvc_status kvc_decode_attention(kvc_cache* c, int layer, const void* q, float sc
 }
 
 kvc_status kvc_decode_attention_layers(kvc_cache* c, int first, int n_layers, const void* q, int64_t q_layer_stride,
-                                       float scale, float* out, int64_t out_layer_stride, void* stream) {
+                                       float scale, float* out, int64_t out_layer_stride, void* stream_) {
   if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
   if (n_layers < 0 || first < 0 || first + n_layers > c->cfg.M)
     return fail(KVC_ERR_INVALID_ARG, "layers [%d, %d) out of range [0, %d)", first, first + n_layers, c->cfg.M);
-  if (n_layers > 0 && (!q || !out)) return fail(KVC_ERR_INVALID_ARG, "q/out are NULL");
+  if (n_layers == 0) return ok();
   const int64_t need = (int64_t)c->cfg.b * c->cfg.H * c->cfg.d_head;
   if (n_layers > 1 && (q_layer_stride < need || out_layer_stride < need))
     return fail(KVC_ERR_INVALID_ARG, "layer strides (%lld, %lld) below one layer's %lld elements",
                 (long long)q_layer_stride, (long long)out_layer_stride, (long long)need);
+  kvc_status st = decode_check(c, first, n_layers, q, scale, out);
+  if (st != KVC_OK) return st;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  st = c->ensure_cuda(stream);
+  if (st != KVC_OK) return st;
+  if (n_layers > 1) {
+    // balanced segments: every layer's in one launch (no per-launch prologue and drain per layer)
+    kvc::DecodeArgs a = decode_args(c, first, q, scale, out);
+    a.n_layers = n_layers;
+    a.q_layer_stride = q_layer_stride;
+    a.out_layer_stride = out_layer_stride;
+    int grid = 0;
+    kvc::DecodePlan plan{-1, 0, 0, 0};
+    cudaError_t e = kvc::launch_decode(c->geom(), c->stat(), c->bufs(), a, c->num_sms, stream, &grid, &plan);
+    if (e == cudaSuccess) {
+      c->last_plan = plan;
+      c->launches += grid > 0 ? 1 : 0;
+      c->last_was_decode = true;
+      return ok();
+    }
+    if (e != cudaErrorNotSupported) return cuda_fail(e, "decode kernel (layers)");
+  }
+  // unbalanced segments (split over a wave of warps per layer): one launch per layer, in order
   const uint16_t* qp = static_cast<const uint16_t*>(q);
   for (int i = 0; i < n_layers; ++i) {
-    kvc_status st = kvc_decode_attention(c, first + i, qp + i * q_layer_stride, scale, out + i * out_layer_stride, stream);
+    st = kvc_decode_attention(c, first + i, qp + i * q_layer_stride, scale, out + i * out_layer_stride, stream);
     if (st != KVC_OK) return st;
   }
   return ok();
@@ -825,15 +883,9 @@ kvc_status kvc_decode_attention_layers(kvc_cache* c, int first, int n_layers, co
 
 kvc_status kvc_decode_attention_static_scratch(kvc_cache* c, int layer, const void* q, float scale, float* out,
                                                void* stream_) {
-  if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
+  kvc_status st0 = decode_check(c, layer, 1, q, scale, out);
+  if (st0 != KVC_OK) return st0;
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
-  if (layer < 0 || layer >= c->cfg.M) return fail(KVC_ERR_INVALID_ARG, "layer %d out of range", layer);
-  if (!q || !out) return fail(KVC_ERR_INVALID_ARG, "q/out are NULL");
-  if (!std::isfinite(scale)) return fail(KVC_ERR_INVALID_ARG, "scale is not finite");
-  if (layer >= c->layers_done) return fail(KVC_ERR_STATE, "layer %d of the last tokens is not written yet", layer);
-  if (!c->cuda_ready) return fail(KVC_ERR_STATE, "nothing appended yet");
-  if (!c->decode_ok) return fail(KVC_ERR_STATE, "%s", c->decode_err.c_str());
-  if (c->R <= 0) return fail(KVC_ERR_STATE, "no sequence has a token to query");
   // split-K partials for every possible worker and segment, then one arrival counter per segment
   const size_t segs = (size_t)c->cfg.b * c->cfg.H;
   const size_t part_bytes = align_up(4 * ((size_t)kvc::kMaxDecodeWorkers + segs) * (size_t)(c->cfg.d_head + 4), 256);
@@ -1080,6 +1132,22 @@ kvc_status kvc_check_bounded_wait(kvc_cache* c, uint64_t limit_ns, void* stream_
 }
 
 int64_t kvc_launch_count(const kvc_cache* c) { return c ? c->launches : 0; }
+
+kvc_status kvc_set_compaction_timing(kvc_cache* c, int enable) {
+  if (!c) return fail(KVC_ERR_INVALID_ARG, "cache is NULL");
+  c->time_compaction = enable != 0;
+  return ok();
+}
+
+kvc_status kvc_last_compaction_ms(kvc_cache* c, float* scan_ms, float* move_ms) {
+  if (!c || !scan_ms || !move_ms) return fail(KVC_ERR_INVALID_ARG, "cache or outputs are NULL");
+  if (!c->timed_compaction) return fail(KVC_ERR_STATE, "the last compaction was not timed");
+  cudaError_t e = cudaEventSynchronize(c->cev[2]);
+  if (e == cudaSuccess) e = cudaEventElapsedTime(scan_ms, c->cev[0], c->cev[1]);
+  if (e == cudaSuccess) e = cudaEventElapsedTime(move_ms, c->cev[1], c->cev[2]);
+  if (e != cudaSuccess) return cuda_fail(e, "compaction timing events");
+  return ok();
+}
 
 kvc_status kvc_last_decode_plan(const kvc_cache* c, int32_t* plan) {
   if (!c || !plan) return fail(KVC_ERR_INVALID_ARG, "NULL argument");

@@ -305,7 +305,8 @@ def test_local_attention_fifo_cache(ratio):
 
 
 def test_multi_layer_decode_call_equals_per_layer_calls():
-    """kvc_decode_attention_layers launches exactly the per-layer decodes: identical outputs."""
+    """kvc_decode_attention_layers over balanced segments is one launch in which every segment is
+    processed whole with the per-layer launches' tile shape: identical outputs."""
     w = wl.opt13b(b=3, L=400, M=3)
     run = harness.Runner(w, 2)
     run.load_prompt()
@@ -314,8 +315,10 @@ def test_multi_layer_decode_call_equals_per_layer_calls():
     one = torch.full((w.M, w.b, w.H, w.d), float("nan"), dtype=torch.float32, device="cuda")
     for m in range(w.M):
         kvc.kvc_decode_attention(run.cache.handle, m, inp.q[m], w.scale, one[m])
+    l0 = run.cache.launch_count
     many = run.cache.decode_attention_layers(inp.q, w.scale)
     torch.cuda.synchronize()
+    assert run.cache.launch_count == l0 + 1
     assert torch.equal(one, many)
     # a run of layers in the middle, with padded strides
     n = w.b * w.H * w.d
@@ -326,4 +329,91 @@ def test_multi_layer_decode_call_equals_per_layer_calls():
     torch.cuda.synchronize()
     assert torch.equal(opad[1:, :n], one[1:].reshape(2, n))
     assert torch.isnan(opad[0]).all()
+    assert run.cache.device_status() == 0
+
+
+def _layers_without_some_tokens(b, M, L=192, dead=lambda s: s % 3 == 1):
+    """An OPT-1.3B-shaped cache of M layers whose `dead` sequences hold no token; the prompt spans of
+    the others are freed.  Returns the runner, the live sequences and every layer's queries at the
+    last prompt token."""
+    w = wl.opt13b(b=b, L=L, M=M)
+    run = harness.Runner(w, steps=1)
+    live = [s for s in range(b) if not dead(s)]
+    n_new = np.array([0 if dead(s) else L for s in range(b)], np.int32)
+    kinds = np.concatenate([w.prompt_kinds[s] for s in live])
+    N = L * len(live)
+    k = torch.empty(M, N * w.H * w.d, dtype=torch.float16, device="cuda")
+    v = torch.empty_like(k)
+    tok_t = torch.from_numpy(np.tile(np.arange(L, dtype=np.int32), len(live))).cuda()
+    tok_s = torch.from_numpy(np.repeat(np.int32(live), L)).cuda()
+    for m in range(M):
+        run._fill(synth.K_TENSOR, m, tok_t, tok_s, k[m], run.kv_scale)
+        run._fill(synth.V_TENSOR, m, tok_t, tok_s, v[m], run.kv_scale)
+    run.cache.append(k, v, n_new, kinds)
+    run.cache.compress_spans([s for s in live for _ in w.prompt_spans[s]],
+                             [a for s in live for a, _ in w.prompt_spans[s]],
+                             [c for s in live for _, c in w.prompt_spans[s]])
+    q = torch.empty(M, b, w.H, w.d, dtype=torch.float16, device="cuda")
+    for m in range(M):
+        run._fill(synth.Q_TENSOR, m, torch.full((b,), L - 1, dtype=torch.int32, device="cuda"),
+                  torch.arange(b, dtype=torch.int32, device="cuda"), q[m], run.q_scale)
+    return w, run, live, q
+
+
+@pytest.mark.parametrize("b", [53, 61])
+def test_fused_layers_several_segments_per_warp_with_empty_sequences(b):
+    """One launch over five layers with more segments than a wave of warps holds: each warp takes k
+    consecutive whole segments and skips the sequences that hold no token.  With a prime b the 32 b
+    segments of a layer are a multiple of k only when k is a power of two, so workers' runs of
+    segments cross from one layer to the next.  Every live output against the oracle; the empty
+    sequences' outputs untouched."""
+    M = 5
+    w, run, live, q = _layers_without_some_tokens(b, M)
+    fused = torch.full((M, b, w.H, w.d), float("nan"), dtype=torch.float32, device="cuda")
+    l0 = run.cache.launch_count
+    run.cache.decode_attention_layers(q, w.scale, fused)
+    torch.cuda.synchronize()
+    assert run.cache.launch_count == l0 + 1
+    plan = run.cache.last_decode_plan
+    assert plan["mode"] == 3, plan
+    one = torch.full_like(fused, float("nan"))
+    for m in range(M):
+        kvc.kvc_decode_attention(run.cache.handle, m, q[m], w.scale, one[m])
+    torch.cuda.synchronize()
+    o, o1 = fused.cpu().numpy(), one.cpu().numpy()
+    dead = [s for s in range(b) if s not in live]
+    assert np.isnan(o[:, dead]).all() and np.isnan(o1[:, dead]).all()
+    for m in range(M):
+        ref = ow.expected_decode(w, 0, m, live)  # queries at the last prompt token, spans freed
+        compare(o[m][live], ref, f"fused layer {m}")
+        compare(o1[m][live], ref, f"per-layer layer {m}")
+    assert run.cache.device_status() == 0
+
+
+def test_fused_layers_fall_back_to_per_layer_launches_when_unbalanced():
+    """Unbalanced segments are split over a wave of warps (stream-K) one layer per launch: the
+    multi-layer call makes M launches and matches the per-layer calls bit for bit."""
+    w = dataclasses.replace(wl.opt13b(b=2, L=64, M=3), name="long-short")
+    k_long, s_long = wl.block_kinds(3000, 32)
+    k_short, s_short = wl.block_kinds(70, 8)
+    w.prompt_kinds = [k_long, k_short]
+    w.prompt_spans = [s_long, s_short]
+    run = harness.Runner(w, 3)
+    run.load_prompt()
+    out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device="cuda")
+    run.step(run.make_step_inputs(0), out)  # a <CL>: its query sees one row, balanced by itself
+    inp = run.make_step_inputs(1)           # a normal token inside the open span
+    run.append_only(inp)
+    one = torch.full((w.M, w.b, w.H, w.d), float("nan"), dtype=torch.float32, device="cuda")
+    for m in range(w.M):
+        kvc.kvc_decode_attention(run.cache.handle, m, inp.q[m], w.scale, one[m])
+    l0 = run.cache.launch_count
+    many = run.cache.decode_attention_layers(inp.q, w.scale)
+    torch.cuda.synchronize()
+    assert run.cache.launch_count == l0 + w.M
+    assert run.cache.last_decode_plan["mode"] == 0
+    assert torch.equal(one, many)
+    o = many.cpu().numpy()
+    for m in range(w.M):
+        compare(o[m], ow.expected_decode(w, 2, m, [0, 1]), f"layer {m}")
     assert run.cache.device_status() == 0
