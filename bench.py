@@ -2,9 +2,12 @@
 
 One step = one pass of the whole hot path over a batch: append the new token's K/V rows (all layers),
 single-query decode attention for every layer over the kept rows, and compaction of the span a <CR>
-just closed.  Workload (default): the OPT-1.3B-shaped cache (M=24, H=32, d_head=64, fp16, b=16,
-prompt 2048 with 32 of every 64 tokens enclosed, a span closed and freed every 33 generated tokens),
-seeded synthetic inputs already resident in HBM.  Every step reads ~3.1 GB, far more than L2.
+just closed.  Workload (default): the ragged stress cache, the largest one that fits one GPU (M=24,
+H=32, d_head=64, fp16, b=128, prompts of U[256, 8192] tokens with half of them enclosed in sampled
+spans, each sequence opening and closing one span during decode), seeded synthetic inputs already
+resident in HBM.  Every step reads ~50 GB, far more than L2.  Beside the headline, the decode and
+compaction roofline fractions of the OPT-1.3B-, OPT-2.7B- and 3B-rotary-shaped caches are measured in
+the same run (`per_workload`).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl kvc|reference]
 
@@ -38,7 +41,12 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=128)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--workload", default="opt1.3b")
+    ap.add_argument("--workload", default="ragged",
+                    help="headline workload (default: the ragged stress cache, the largest single-GPU one)")
+    ap.add_argument("--per-workload", default="opt1.3b,opt2.7b,rope3b_I19,rope3b_I32,rope3b_I45",
+                    help="workloads whose decode and compaction fractions are reported beside the headline "
+                         "('' for none)")
+    ap.add_argument("--per-workload-steps", type=int, default=16)
     ap.add_argument("--impl", default="kvc", choices=["kvc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -217,24 +225,27 @@ class ClockSampler:
 # ------------------------------------------------------------------------------------------------
 
 class OracleSample:
-    """Full-length masked decode of one layer for every sequence of the workload, by the fp64 oracle on
-    the host cores.  K/V of that layer are generated once for the whole capacity (not timed)."""
+    """Full-length masked decode of a set of layers for every sequence of the workload, by the fp64
+    oracle on the host cores.  K/V of those layers are generated once for the whole capacity (not
+    timed)."""
 
-    def __init__(self, w, steps_total: int, layer: int = 0):
+    def __init__(self, w, steps_total: int, layers=(0,)):
         import oracle
         import oracle.workload as ow
 
-        self.oracle, self.ow, self.w, self.layer = oracle, ow, w, layer
-        self.K, self.V = [], []
-        for s in range(w.b):
-            T = int(w.prompt_len[s]) + steps_total
-            K, V = ow.kv_bits(w, layer, s, T)
-            self.K.append(K)
-            self.V.append(V)
+        self.oracle, self.ow, self.w, self.layers = oracle, ow, w, list(layers)
+        self.K, self.V = {}, {}
+        for m in self.layers:
+            self.K[m], self.V[m] = [], []
+            for s in range(w.b):
+                T = int(w.prompt_len[s]) + steps_total
+                K, V = ow.kv_bits(w, m, s, T)
+                self.K[m].append(K)
+                self.V[m].append(V)
         self.threads = oracle.max_threads()
 
-    def time_step(self, g: int) -> float:
-        """Seconds the oracle takes for layer `layer` of decode step g (query = generated token g)."""
+    def time_step(self, g: int, layer: int = 0) -> float:
+        """Seconds the oracle takes for one layer of decode step g (query = generated token g)."""
         w, ow = self.w, self.ow
         kinds_l, pos_l, K_l, V_l, q_l = [], [], [], [], []
         for s in range(w.b):
@@ -242,9 +253,9 @@ class OracleSample:
             T = kinds.size
             kinds_l.append(kinds)
             pos_l.append(pos)
-            K_l.append(np.ascontiguousarray(self.K[s][:, :T]))
-            V_l.append(np.ascontiguousarray(self.V[s][:, :T]))
-            q_l.append(ow.q_bits(w, self.layer, s, T - 1))
+            K_l.append(np.ascontiguousarray(self.K[layer][s][:, :T]))
+            V_l.append(np.ascontiguousarray(self.V[layer][s][:, :T]))
+            q_l.append(ow.q_bits(w, layer, s, T - 1))
         q = np.stack(q_l)
         t0 = time.perf_counter()
         self.oracle.masked_decode(kinds_l, pos_l, K_l, V_l, q, w.dtype, w.scale, rot=w.rotary_dim,
@@ -272,6 +283,11 @@ def cpu_baseline(w, steps_total: int, budget_s: float):
                       "K/V generation not timed"}
 
 
+# All layers of a step are timed when their K/V history fits this many bytes of host memory; beyond
+# it (the 2.7B- and 3B-shaped caches, the ragged one) one layer per step is timed and scaled by M.
+REFERENCE_ALL_LAYERS_BYTES = 8 << 30
+
+
 # ------------------------------------------------------------------------------------------------
 # arms
 # ------------------------------------------------------------------------------------------------
@@ -285,26 +301,47 @@ def dist_setup(n_gpus: int):
     return rank, world, local
 
 
+def reference_layers(w, steps_total: int):
+    """Layers the reference arm times per step, and the bytes of the whole K/V history (all layers)."""
+    hist_bytes = 2 * 2 * w.M * w.H * w.d * int((w.prompt_len + steps_total).sum())
+    return (list(range(w.M)) if hist_bytes <= REFERENCE_ALL_LAYERS_BYTES else [0]), hist_bytes
+
+
 def run_reference(args, w):
+    """The reference arm: the fp64 oracle on the host cores, full-length masked decode of every
+    sequence under the paper's mask.  A step times every layer when the whole K/V history fits
+    REFERENCE_ALL_LAYERS_BYTES of host memory, else layer 0 alone (layers are independent and
+    processed identically) and the step's all-layer time is extrapolated by M.  ms_per_step is the
+    host time the timed layers took, so ms_per_step x steps is what ran; with a sampled step the line
+    says so (extrapolated, layers_timed_per_step) and gives the extrapolated step time beside it."""
     rank, world, _ = dist_setup(args.gpus)
     if rank != 0:
         return
     steps_total = args.warmup + args.steps
-    samp = OracleSample(w, steps_total)
+    layers, hist_bytes = reference_layers(w, steps_total)
+    samp = OracleSample(w, steps_total, layers)
     for g in range(args.warmup):
-        samp.time_step(g)
-    times = [samp.time_step(args.warmup + k) for k in range(args.steps)]
-    per_layer = sum(times) / len(times)
+        samp.time_step(g, layers[0])
+    step_s = []
+    for k in range(args.steps):
+        step_s.append(sum(samp.time_step(args.warmup + k, m) for m in layers))
+    per_layer = sum(step_s) / (len(step_s) * len(layers))
     value = samp.tokens_per_s(per_layer)
+    sampled = len(layers) < w.M
+    what = (f"every layer ({w.M})" if not sampled else
+            f"layer 0 of {w.M} (the {hist_bytes / 2**30:.0f} GiB K/V history does not fit the host budget), "
+            f"scaled by M")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_layer * w.M * 1e3,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": sum(step_s) / len(step_s) * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded counter-based generator)",
         "config": workload_config(w),
+        "extrapolated": sampled, "layers_timed_per_step": len(layers),
+        "ms_per_step_all_layers": per_layer * w.M * 1e3,
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": samp.threads, "kind": "oracle",
-                         "sample": f"each step: fp64 oracle full-length masked decode of layer 0 for all {w.b} "
-                                   f"sequences, scaled by M={w.M}; K/V generation not timed"},
+                         "sample": f"each step: fp64 oracle full-length masked decode of all {w.b} sequences, "
+                                   f"{what}; K/V generation not timed"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -334,16 +371,26 @@ def aggregate(local_tokens: int, local_elapsed: float, device=None):
 
 def time_prompt_compaction(run, w):
     """Frees every prompt span in one go (one compaction over all sequences and layers) and reports
-    the row-move bandwidth: bytes = 2 (read + write) x moved rows x row bytes x M x 2 (K, V) x H."""
+    the row-move bandwidth: bytes = 2 (read + write) x moved rows x row bytes x M x 2 (K, V) x H,
+    over the device time of the two kernels (the library's events before the scan, between the
+    kernels and after the row moves).  call_ms is the whole call measured from an idle stream: it
+    also holds the host's planning of the compaction, which a decode loop overlaps with the GPU."""
     import torch
 
+    import paper_2310_08152_gb300 as kvc
+
+    kvc.kvc_set_compaction_timing(run.cache.handle, True)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
     e0.record()
     run.compress_prompt()
     e1.record()
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1)
+    call_ms = e0.elapsed_time(e1)
+    scan_ms = move_ms = None
+    if any(w.prompt_spans[s] for s in range(w.b)):  # else nothing was compacted (no spans)
+        scan_ms, move_ms = kvc.kvc_last_compaction_ms(run.cache.handle)
+    kvc.kvc_set_compaction_timing(run.cache.handle, False)
     ln = run.cache.lengths()[0]
     moved = 0
     for s in range(w.b):
@@ -352,10 +399,14 @@ def time_prompt_compaction(run, w):
             moved += int(ln[s]) - first
     nbytes = 2 * moved * w.d * 2 * w.M * 2 * w.H
     peak, kind = measured_hbm_peak()
-    gbs = nbytes / (ms * 1e-3) / 1e9 if ms > 0 else None
+    ms = (scan_ms + move_ms) if scan_ms is not None else None
+    gbs = nbytes / (ms * 1e-3) / 1e9 if ms else None
+    move_gbs = nbytes / (move_ms * 1e-3) / 1e9 if move_ms else None
     return {"kernels": "compact_scan_kernel + compact_move_kernel", "moved_rows_per_stream": moved,
-            "bytes": nbytes, "ms": ms, "achieved": gbs, "peak": peak, "unit": "GB/s",
-            "frac": (gbs / peak) if gbs else None, "peak_kind": kind}
+            "bytes": nbytes, "ms": ms, "scan_ms": scan_ms, "move_ms": move_ms, "call_ms": call_ms,
+            "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": (gbs / peak) if gbs else None,
+            "frac_of_8tbs": gbs / 8000.0 if gbs else None,
+            "move_frac": (move_gbs / peak) if move_gbs else None, "peak_kind": kind}
 
 
 def time_prompt_write_time_freeing(w, steps_total, dev):
@@ -495,12 +546,113 @@ def run_capacity_sweep(args):
             torch.cuda.empty_cache()
 
 
+def timed_decode_steps(run, w, inputs, warmup: int, steps: int, world: int = 1, clocks=None):
+    """Warm-up steps through the harness, then `steps` timed decode steps in a lean loop: device
+    pointers are computed up front and the entry points are called directly, so the host enqueues
+    faster than the GPU drains.  Each step: append the token (all layers), decode every layer in one
+    kvc_decode_attention_layers call (one launch when the segments are balanced, else one per layer),
+    free the span a <CR> closed.  An event pair around each step's decode call times the decode."""
+    import torch
+    import torch.distributed as dist
+
+    import paper_2310_08152_gb300 as kvc
+
+    dev = run.device
+    out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()
+    for g in range(warmup):
+        run.step(inputs[g], out)
+    dec = kvc.lib().kvc_decode_attention_layers
+    stream_h = torch.cuda.current_stream().cuda_stream
+    handle = run.cache.handle
+    n = w.b * w.H * w.d
+    q_ptrs = [inputs[g].q.data_ptr() for g in range(warmup + steps)]
+    out_ptr = out.data_ptr()
+    ones = np.ones(w.b, np.int32)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    bytes_per_step, dec_launches = [], 0
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    launches0 = run.cache.launch_count
+    if clocks is not None:
+        clocks.start()
+    t_start.record()
+    for k in range(steps):
+        g = warmup + k
+        inp = inputs[g]
+        run.cache.append(inp.kv_k, inp.kv_v, ones, inp.kinds)
+        # decode bytes of this step are fixed once the token is appended: computed from the host lengths
+        bytes_per_step.append(run.decode_bytes() * w.M)
+        l0 = run.cache.launch_count
+        ev[k][0].record()
+        rc = dec(handle, 0, w.M, q_ptrs[g], n, w.scale, out_ptr, n, stream_h)
+        ev[k][1].record()
+        if rc:
+            raise kvc.KvcError(rc, kvc.lib().kvc_last_error().decode())
+        dec_launches += run.cache.launch_count - l0
+        seq, cl, cr = run.step_spans(inp.kinds)
+        run.g += 1
+        if seq:
+            run.cache.compress_spans(seq, cl, cr)
+    t_end.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop() if clocks is not None else None
+    launches = run.cache.launch_count - launches0
+    elapsed = t_start.elapsed_time(t_end) / 1e3
+    dec_us = [e0.elapsed_time(e1) * 1e3 for e0, e1 in ev]
+    dec_total_s = sum(dec_us) / 1e6
+    achieved = sum(bytes_per_step) / dec_total_s / 1e9
+    peak, peak_kind = measured_hbm_peak()
+    plan = run.cache.last_decode_plan
+    return {"elapsed": elapsed, "tokens": w.b * steps, "launches": launches, "dec_launches": dec_launches,
+            "dec_total_s": dec_total_s, "dec_us": dec_us, "bytes": sum(bytes_per_step), "achieved": achieved,
+            "peak": peak, "peak_kind": peak_kind, "plan": plan, "clocks": clk}
+
+
+PLAN_NAMES = ["stream-K", "warp per segment (wide)", "warp per segment (narrow)", "whole segments, several per warp"]
+
+
+def plan_record(plan, launches_per_step: float):
+    return {"mode": PLAN_NAMES[plan["mode"]] if plan["mode"] >= 0 else None, "warps": plan["workers"],
+            "tile_rows": plan["tile_rows"], "stages": plan["stages"], "launches_per_step": launches_per_step}
+
+
+def measure_workload(name: str, dev, steps: int, warmup: int = 3):
+    """Decode and compaction roofline fractions of one more workload, measured the way the headline is
+    (a shorter timed window): prompt appended, freed in one compaction (timed), then timed steps."""
+    import torch
+
+    import harness
+    from synth import workloads as wl
+
+    w = wl.by_name(name)
+    run = harness.Runner(w, warmup + steps, device=dev)
+    run.load_prompt(compress=False)
+    comp = time_prompt_compaction(run, w)
+    inputs = [run.make_step_inputs(g) for g in range(warmup + steps)]
+    r = timed_decode_steps(run, w, inputs, warmup, steps)
+    status = run.cache.device_status()
+    del inputs, run
+    torch.cuda.empty_cache()
+    n_launch = max(1, r["dec_launches"])
+    return {"workload": name, "tokens_per_s": r["tokens"] / r["elapsed"], "steps": steps,
+            "decode": {"achieved": r["achieved"], "peak": r["peak"], "unit": "GB/s",
+                       "frac": r["achieved"] / r["peak"], "frac_of_8tbs": r["achieved"] / 8000.0,
+                       "peak_kind": r["peak_kind"], "bytes_per_launch_mean": r["bytes"] / n_launch,
+                       "launch_us_mean": r["dec_total_s"] / n_launch * 1e6,
+                       "plan": plan_record(r["plan"], r["dec_launches"] / steps)},
+            "compaction": {k: comp[k] for k in ("bytes", "ms", "scan_ms", "move_ms", "call_ms", "achieved", "frac",
+                                                "frac_of_8tbs", "move_frac")},
+            "device_status": status}
+
+
 def run_kvc(args, w):
     import torch
     import torch.distributed as dist
 
     import harness
-    import paper_2310_08152_gb300 as kvc
 
     rank, world, local = dist_setup(args.gpus)
     torch.cuda.set_device(local)
@@ -523,59 +675,10 @@ def run_kvc(args, w):
     else:
         prefill = [time_prompt_prefill(w, steps_total, dev, blk) for blk in (0, 512)]
     inputs = [run.make_step_inputs(g) for g in range(steps_total)]
-    out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device=dev)
-    torch.cuda.synchronize()
-    for g in range(args.warmup):
-        run.step(inputs[g], out)
-    # Lean timed loop: device pointers are computed up front and the decode entry point is called
-    # directly, so the host enqueues faster than the GPU drains (no idle gaps from Python overhead).
-    dec = kvc.lib().kvc_decode_attention
-    stream_h = torch.cuda.current_stream().cuda_stream
-    handle = run.cache.handle
-    q_ptrs = [[inputs[g].q[m].data_ptr() for m in range(w.M)] for g in range(steps_total)]
-    out_ptrs = [out[m].data_ptr() for m in range(w.M)]
-    ones = np.ones(w.b, np.int32)
-    # one (start, end) event pair per step around its M decode launches
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    bytes_per_step = []
-    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    clocks = ClockSampler(local)
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    launches0 = run.cache.launch_count
-    clocks.start()
-    t_start.record()
-    for k in range(args.steps):
-        g = args.warmup + k
-        inp = inputs[g]
-        run.cache.append(inp.kv_k, inp.kv_v, ones, inp.kinds)
-        # decode bytes of this step are fixed once the token is appended: computed from the host lengths
-        bytes_per_step.append(run.decode_bytes())
-        qp = q_ptrs[g]
-        ev[k][0].record()
-        for m in range(w.M):
-            rc = dec(handle, m, qp[m], w.scale, out_ptrs[m], stream_h)
-            if rc:
-                raise kvc.KvcError(rc, kvc.lib().kvc_last_error().decode())
-        ev[k][1].record()
-        seq, cl, cr = run.step_spans(inp.kinds)
-        run.g += 1
-        if seq:
-            run.cache.compress_spans(seq, cl, cr)
-    t_end.record()
-    torch.cuda.synchronize()
-    clk = clocks.stop()
-    launches = run.cache.launch_count - launches0
-    elapsed = t_start.elapsed_time(t_end) / 1e3
-    tokens, elapsed = aggregate(w.b * args.steps, elapsed, dev)
+    r = timed_decode_steps(run, w, inputs, args.warmup, args.steps, world, ClockSampler(local))
+    tokens, elapsed = aggregate(r["tokens"], r["elapsed"], dev)
     value = tokens / elapsed
-    plan = run.cache.last_decode_plan
-    dec_total_s = sum(e0.elapsed_time(e1) for e0, e1 in ev) / 1e3
-    dec_bytes_total = sum(b * w.M for b in bytes_per_step)
-    achieved = dec_bytes_total / dec_total_s / 1e9
-    peak, peak_kind = measured_hbm_peak()
-    launches_decode = args.steps * w.M
+    n_launch = max(1, r["dec_launches"])
     status = run.cache.device_status()
     del inputs, run
     torch.cuda.empty_cache()
@@ -585,29 +688,37 @@ def run_kvc(args, w):
     if not args.no_e2e:
         e2e = run_e2e(args, w, dev, world)
 
+    # ---------------- the other workloads' roofline fractions (rank 0) ----------------
+    per_workload = []
+    if rank == 0 and args.per_workload:
+        for name in [x for x in args.per_workload.split(",") if x and x != w.name]:
+            per_workload.append(measure_workload(name, dev, args.per_workload_steps))
+
     if rank == 0:
+        dec_us = sorted(r["dec_us"])
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": elapsed / args.steps * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
             "data": "synthetic (seeded counter-based generator; no dataset or weights)",
             "config": workload_config(w),
-            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "peak_kind": peak_kind,
+            "roofline": {"bound": "hbm", "achieved": r["achieved"], "peak": r["peak"], "unit": "GB/s",
+                         "frac": r["achieved"] / r["peak"], "frac_of_8tbs": r["achieved"] / 8000.0,
+                         "peak_kind": r["peak_kind"],
                          "kernel": "decode_kernel (split-K single-query attention + log-sum-exp combine)",
                          "traffic": recorded_traffic(w.name),
-                         "bytes_per_launch_mean": dec_bytes_total / launches_decode,
-                         "launch_us_mean": dec_total_s / launches_decode * 1e6},
-            "decode_plan": {"mode": ["stream-K", "warp per segment (wide)", "warp per segment (narrow)", "whole segments, several per warp"][plan["mode"]]
-                            if plan["mode"] >= 0 else None, "warps": plan["workers"],
-                            "tile_rows": plan["tile_rows"], "stages": plan["stages"]},
-            "decode_share_of_step": dec_total_s / elapsed,
+                         "bytes_per_launch_mean": r["bytes"] / n_launch,
+                         "launch_us_mean": r["dec_total_s"] / n_launch * 1e6},
+            "decode_plan": plan_record(r["plan"], r["dec_launches"] / args.steps),
+            "decode_us_per_step": {"min": dec_us[0], "median": statistics.median(dec_us), "max": dec_us[-1]},
+            "decode_share_of_step": r["dec_total_s"] / r["elapsed"],
             "compaction": compaction,
             "prompt_write_time_freeing": prompt_free,
             "prefill": prefill,
-            "gpu_launches": launches,
+            "per_workload": per_workload,
+            "gpu_launches": r["launches"],
             "device_status": status,
-            "clocks": clk,
+            "clocks": r["clocks"],
             "e2e": e2e,
         }
         if not args.no_cpu_baseline:

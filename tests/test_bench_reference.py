@@ -30,6 +30,22 @@ def _check_line(line, gpus):
     e = line["e2e"]
     assert e["value"] == line["value"] and e["unit"] == line["unit"]
     assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
+    # tiny's one layer is timed whole every step: the step time is what ran, and the value follows from it
+    assert line["extrapolated"] is False and line["layers_timed_per_step"] == 1
+    assert abs(line["value"] - 2 / (line["ms_per_step"] / 1e3)) <= 1e-9 * line["value"]
+
+
+def test_reference_arm_times_every_layer_where_the_history_fits():
+    """The OPT-1.3B-shaped history (~7 GB of K/V) is timed layer by layer in full; the ragged one
+    (~100 GB) is sampled at layer 0 and flagged as extrapolated."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from synth import workloads as wl
+
+    layers, nbytes = bench.reference_layers(wl.opt13b(), 25)
+    assert layers == list(range(24)) and nbytes < bench.REFERENCE_ALL_LAYERS_BYTES
+    layers, nbytes = bench.reference_layers(wl.ragged(), 25)
+    assert layers == [0] and nbytes > 50e9
 
 
 def test_reference_arm_single_rank():

@@ -50,7 +50,68 @@ def test_full_opt27b_shaped():
 
 @pytest.mark.parametrize("interior", [19, 32, 45])
 def test_full_rope3b_shaped(interior):
-    _full(wl.rope3b(interior), 8, check_at={0, 7}, rope=True)
+    # all 128 steps of the workload: the query positions run up to 2048 + 127 over the full cache
+    _full(wl.rope3b(interior), 128, check_at={0, 64, 127}, rope=True)
+
+
+# --------------------------------------------------------------------------
+# The capacity / throughput sweep's shapes (Sec. 4.3, App. C): RedPajama-3B-shaped caches (H = 32,
+# d_head = 80, fp16, RoPE), an 800-token prefix at r = 0.9 with the <CL> at offset 0 of every
+# 64-token block, ingested with write-time freeing, and the sweep's largest batch, b = 4096: 131,072
+# (sequence, head) segments per layer.  Two layers stand for the model's 32 (layers are independent
+# and processed identically); the bench's step calls decode all of them in one launch.
+# --------------------------------------------------------------------------
+
+def _sweep_run(w, steps, seqs, rng):
+    kept = [int(w.prompt_len[s]) - sum(c - a for a, c in w.prompt_spans[s]) for s in range(w.b)]
+    run = harness.Runner(w, steps, capacity=np.asarray(kept, np.int64) + steps)
+    run.load_prompt(mode="free")
+    assert int(run.cache.lengths()[0].sum()) == sum(kept)
+    out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device=run.device)
+    plans = []
+    for g in range(steps):
+        inp = run.make_step_inputs(g)
+        out.fill_(float("nan"))
+        run.step(inp, out)
+        plans.append(run.cache.last_decode_plan)
+        torch.cuda.synchronize()
+        o = out.cpu().numpy()
+        assert np.all(np.isfinite(o))
+        if g in (0, steps - 1):
+            for m in range(w.M):
+                compare(o[m][seqs], ow.expected_decode(w, g + 1, m, seqs), f"{w.name} step {g} layer {m}")
+    assert run.cache.device_status() == 0
+    return run, plans
+
+
+def test_capacity_sweep_shapes_b4096():
+    w = wl.throughput_3b(0.9, b=4096, M=2, steps=4)
+    rng = np.random.default_rng(9)
+    seqs = sorted({0, 1, 2047, 4095, *rng.integers(0, 4096, size=6).tolist()})
+    run, plans = _sweep_run(w, 4, seqs, rng)
+    # balanced segments: several whole segments per warp, both layers in one launch
+    assert all(p["mode"] == 3 for p in plans), plans
+
+
+def test_capacity_sweep_shapes_b4096_unbalanced_stream_k():
+    """The same cache with one sequence's prefix ten times longer: the segments are unbalanced, so each
+    layer's rows are split evenly over a full wave of warps (stream-K).  Every warp then covers dozens
+    of whole segments plus split pieces at both ends, and the long sequence's segments are split over
+    several warps and merged by the log-sum-exp combine."""
+    import dataclasses
+
+    w = wl.throughput_3b(0.9, b=4096, M=1, steps=3)
+    k_long, s_long = wl.block_kinds(8000, 58, cl_off=0)
+    kinds = list(w.prompt_kinds)
+    spans = list(w.prompt_spans)
+    kinds[1], spans[1] = k_long, s_long
+    w = dataclasses.replace(w, prompt_kinds=kinds, prompt_spans=spans, name="throughput3b_r0.90_long1")
+    rng = np.random.default_rng(10)
+    seqs = sorted({0, 1, 2, 4095, *rng.integers(0, 4096, size=6).tolist()})
+    run, plans = _sweep_run(w, 3, seqs, rng)
+    assert all(p["mode"] == 0 for p in plans), plans
+    rows = int(run.attended_rows().sum()) * w.H
+    assert rows // plans[-1]["workers"] > 20 * 110  # dozens of ~100-row segments per warp
 
 
 def test_full_ragged():

@@ -4,8 +4,8 @@ Some callers run where new device allocations are not allowed -- inside a fixed,
 pool, or under an allocator that forbids cudaMalloc once serving has started -- so they cannot
 give the decode a scratch buffer of its own.  This entry point keeps its split-K scratch in a
 file-scope device array of the library instead.  Its results must equal those of the regular entry
-point, on two calls in a row (the array keeps the previous call's contents, so each call must start
-from a clean state).  Collected last on purpose: a failure here leaves every other test already run.
+point bit for bit, on two calls in a row (the array keeps the previous call's contents, so each call
+must start from a clean state), and the calls must allocate no device memory.  Collected last on purpose: a failure here leaves every other test already run.
 """
 import dataclasses
 
@@ -34,20 +34,31 @@ def _workloads():
 
 @pytest.mark.parametrize("w", _workloads(), ids=lambda w: w.name)
 def test_static_scratch_decode_matches_workspace_decode(w):
+    """Same kernel, same plan, same inputs as kvc_decode_attention: the outputs are equal bit for bit,
+    on two calls in a row, and the calls allocate no device memory."""
     run = harness.Runner(w, steps=2)
     run.load_prompt()
     for g in range(2):
         inp = run.make_step_inputs(g)
         out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device="cuda")
-        run.step(inp, out)  # regular entry point (workspace scratch), then frees closed spans
-        # the query is still the last token: decode it again through the static scratch, twice
+        run.append_only(inp)
+        # the regular entry point (split-K scratch in the cache workspace), layer by layer
+        for m in range(w.M):
+            kvc.kvc_decode_attention(run.cache.handle, m, inp.q[m], w.scale, out[m])
+        alt = torch.full((2, w.M, w.b, w.H, w.d), float("nan"), device="cuda")
+        torch.cuda.synchronize()
+        # the same query through the static scratch, twice; the second time no lookup is left to do
         for rep in range(2):
+            free0, alloc0 = torch.cuda.mem_get_info()[0], torch.cuda.memory_allocated()
             for m in range(w.M):
-                alt = torch.full((w.b, w.H, w.d), float("nan"), device="cuda")
-                kvc.kvc_decode_attention_static_scratch(run.cache.handle, m, inp.q[m], w.scale, alt)
-                torch.cuda.synchronize()
-                compare(alt.cpu().numpy(), out[m].cpu().numpy().astype(np.float64),
-                        f"{w.name} step {g} layer {m} call {rep}")
+                kvc.kvc_decode_attention_static_scratch(run.cache.handle, m, inp.q[m], w.scale, alt[rep, m])
+            torch.cuda.synchronize()
+            if rep == 1:
+                assert torch.cuda.mem_get_info()[0] == free0, "device memory was allocated"
+                assert torch.cuda.memory_allocated() == alloc0
+            assert torch.equal(alt[rep], out), f"{w.name} step {g} call {rep}: not bit-identical"
+        compare(alt[1, 0].cpu().numpy(), out[0].cpu().numpy().astype(np.float64), f"{w.name} step {g}")
+        run.finish_step(inp)  # frees the span a <CR> closed
     assert run.cache.device_status() == 0
 
 
