@@ -17,6 +17,7 @@ shards by sequence with no exchange); value = tokens of all ranks / max time ove
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import math
@@ -53,6 +54,8 @@ def parse():
     ap.add_argument("--e2e-reps", type=int, default=3, help="timed end-to-end windows (median reported)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="budget of the CPU-baseline sample")
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (small profiling runs)")
+    ap.add_argument("--ragged-lengths", default="",
+                    help="LMIN,LMAX: prompt-length range of the ragged workload (small profiling runs)")
     ap.add_argument("--capacity-sweep", action="store_true",
                     help="largest batch under a KV-memory cap per compression ratio, and its throughput")
     ap.add_argument("--caps", default="12,24,180", help="KV-memory caps in GB for --capacity-sweep")
@@ -114,7 +117,10 @@ def recorded_traffic(workload: str):
 
 
 class ClockSampler:
-    """SM clock and clock-event (throttle) reasons sampled every few ms while the timed region runs.
+    """SM clock and clock-event (throttle) reasons sampled every 50 ms while the timed region runs.
+
+    Sampling NVML every 2 ms slowed the end-to-end steps by about 10 % (the GPU's own time, with copies
+    on two more streams); every 50 ms had no measurable effect.
 
     Reads NVML (libnvidia-ml) through ctypes; falls back to `nvidia-smi -lms` when NVML is not
     loadable.  Only reads state; changes nothing on the GPU."""
@@ -122,7 +128,7 @@ class ClockSampler:
     REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
                0x80: "hw_power_brake_slowdown"}
 
-    def __init__(self, gpu_index: int, period_s: float = 0.002):
+    def __init__(self, gpu_index: int, period_s: float = 0.05):
         self.gpu = gpu_index
         self.period = period_s
         self.samples = []
@@ -611,7 +617,8 @@ def timed_decode_steps(run, w, inputs, warmup: int, steps: int, world: int = 1, 
             "peak": peak, "peak_kind": peak_kind, "plan": plan, "clocks": clk}
 
 
-PLAN_NAMES = ["stream-K", "warp per segment (wide)", "warp per segment (narrow)", "whole segments, several per warp"]
+PLAN_NAMES = ["stream-K", "warp per segment (wide)", "warp per segment (narrow)", "whole segments, several per warp",
+              "whole segments cut by rows"]
 
 
 def plan_record(plan, launches_per_step: float):
@@ -838,10 +845,16 @@ def main():
     if args.capacity_sweep:
         run_capacity_sweep(args)
         return
-    w = wl.by_name(args.workload)
+    kw = {}
+    if args.ragged_lengths:
+        if args.workload != "ragged":
+            raise SystemExit("--ragged-lengths applies to the ragged workload only")
+        lmin, lmax = (int(x) for x in args.ragged_lengths.split(","))
+        kw = {"lmin": lmin, "lmax": lmax}
+    w = wl.by_name(args.workload, **kw)
+    if args.ragged_lengths:
+        w = dataclasses.replace(w, name=f"{w.name}-L{lmin}-{lmax}")
     if args.layers:
-        import dataclasses
-
         w = dataclasses.replace(w, M=args.layers, name=f"{w.name}-M{args.layers}")
     if args.prefill_only:
         import torch

@@ -227,11 +227,12 @@ kvc_status kvc_decode_attention(kvc_cache* cache, int layer, const void* q, floa
  * model whose queries for all those layers are ready, as in the paper's throughput setting,
  * Sec. 4.3): layer first + i reads q + i * q_layer_stride elements of the cache dtype and writes
  * out + i * out_layer_stride floats; strides are in elements, each layer's slice laid out as for
- * kvc_decode_attention.  When every (sequence, head) segment holds about as many rows as the others
- * (the longest at most 1.3x the mean), one launch covers every layer's segments, each processed
- * whole by one warp exactly as a per-layer launch with the same tile shape does it; otherwise the
- * layers are launched one by one, in order, on `stream`, and on an error the layers before the
- * failing one have been launched. */
+ * kvc_decode_attention.  One launch covers every layer's segments, each (layer, sequence, head)
+ * segment processed whole by one warp exactly as a per-layer launch with the same tile shape does it,
+ * when the segments hold about as many rows as each other (the longest at most 1.3x the mean) or when
+ * the longest is short beside a warp's even share of all the layers' rows (at most 1/32 of it; the
+ * warps then take runs of whole segments cut by rows).  Otherwise the layers are launched one by one,
+ * in order, on `stream`, and on an error the layers before the failing one have been launched. */
 kvc_status kvc_decode_attention_layers(kvc_cache* cache, int first, int n_layers, const void* q, int64_t q_layer_stride,
                                        float scale, float* out, int64_t out_layer_stride, void* stream);
 
@@ -309,7 +310,8 @@ kvc_status kvc_last_compaction_ms(kvc_cache* cache, float* scan_ms, float* move_
 /* How the last decode launch divided its work (host-side record, no synchronisation):
  * plan[0] = mode (0: the kept rows split evenly over a full wave of warps, split (sequence, head)
  * segments merged by a log-sum-exp combine; 1 / 2: one warp per segment with the wide / narrow
- * shared-memory pipeline; 3: several consecutive whole segments per warp, no combine; -1: nothing
+ * shared-memory pipeline; 3: several consecutive whole segments per warp, no combine; 4: runs of
+ * consecutive whole segments per warp cut by rows, over several layers, no combine; -1: nothing
  * launched yet), plan[1] = warps, plan[2] = rows per tile, plan[3] = pipeline stages per warp. */
 kvc_status kvc_last_decode_plan(const kvc_cache* cache, int32_t* plan);
 

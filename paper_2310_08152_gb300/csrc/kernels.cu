@@ -512,7 +512,9 @@ struct DecodeDev {
   float qscale;  // scale * log2(e)
   unsigned long long limit_ns;
   int kv_before_wait;  // the K/V rows may be streamed before the preceding grid completes
-  int seg_per_worker;  // k > 0: worker w owns segments [w k, w k + k) whole; 0: stream-K split of the rows
+  // k > 0: worker w owns segments [w k, w k + k) whole; -1: worker w owns the whole segments whose
+  // first row lies in its even share of the rows; 0: stream-K split of the rows
+  int seg_per_worker;
 };
 
 // The tiles of a worker: its flat row range [x, hi) of the concatenation over (layer, sequence,
@@ -588,7 +590,7 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
   const int H = g.H;
   const int64_t segs_layer = (int64_t)g.b * H;
   int64_t lo, hi;
-  if (p.seg_per_worker) {  // segments [sg0, sg1) = (layer, s, h) triples in order, each whole
+  if (p.seg_per_worker > 0) {  // segments [sg0, sg1) = (layer, s, h) triples in order, each whole
     // first flat row of segment sg (sg = n_layers * b * H gives the end of the last layer)
     auto seg_row = [&](int64_t sg) {
       const int64_t l = sg / segs_layer, w = sg - l * segs_layer;
@@ -600,6 +602,23 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
     const int64_t sg1 = min(sg0 + p.seg_per_worker, (int64_t)p.n_layers * segs_layer);
     lo = seg_row(sg0);
     hi = seg_row(sg1);
+  } else if (p.seg_per_worker < 0) {
+    // whole segments cut by rows: a segment belongs to the worker whose even share of the flat rows
+    // [w Rt / NW, (w + 1) Rt / NW) holds its first row, so no segment is split and every worker's
+    // rows are within one segment of the even share
+    const int64_t Rt = (int64_t)p.n_layers * p.R;
+    auto seg_at_or_after = [&](int64_t x) {  // first row of the first segment starting at or after x
+      if (x >= Rt) return Rt;
+      const int64_t l = x / p.R, o = x - l * p.R;
+      const int s = seq_of_row(p.P, g.b, H, o, lane);
+      const int64_t a = p.P[s], Lc = p.P[s + 1] - a;
+      const int64_t off = o - (int64_t)H * a;
+      const int64_t h = off / Lc;
+      const int64_t start = l * p.R + (int64_t)H * a + h * Lc;
+      return start == x ? start : start + Lc;
+    };
+    lo = seg_at_or_after((int64_t)wid * Rt / p.NW);
+    hi = seg_at_or_after((int64_t)(wid + 1) * Rt / p.NW);
   } else {
     const int64_t Rt = (int64_t)p.n_layers * p.R;
     lo = (int64_t)wid * Rt / p.NW;
@@ -682,7 +701,7 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
     }
   }
 
-  // raw q of the next piece (and its rotation partner), fetched one tile ahead of its use
+  // raw q of the next piece (and its rotation partner), fetched when the current piece starts
   constexpr int QPL = (D + 31) / 32;
   float qa[QPL], qb[QPL];
   auto fetch_q = [&](int l_, int s_, int h_) {
@@ -760,12 +779,15 @@ __global__ void __launch_bounds__(32, 1) decode_kernel(Geometry g, Static st, De
       l = 0.f;
       piece_whole = (r0 == 0);
       piece_start = false;
-    }
-    if (r0 + n == ci.Lc && ci.x + n < ci.hi) {  // this tile ends the segment: fetch the next piece's q
-      TileIter nx = ci;
-      nx.advance(n, p.P, H, g.b);
-      fetch_q(nx.layer, nx.s, nx.h);
-      if (nx.s != s) dn = p.ds[nx.s];
+      // the next piece's q and sequence state, fetched a whole piece ahead of their use: with short
+      // segments one tile of lead does not cover a global load's latency under full memory traffic
+      const int64_t rest = ci.Lc - r0;  // rows of this segment from here on
+      if (ci.x + rest < ci.hi) {
+        TileIter nx = ci;
+        nx.advance(rest, p.P, H, g.b);
+        fetch_q(nx.layer, nx.s, nx.h);
+        if (nx.s != s) dn = p.ds[nx.s];
+      }
     }
     if (!dead) {
       if (mbar_wait_bounded(&full[stage], (t / C::S) & 1, p.limit_ns)) {
@@ -1044,11 +1066,25 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   // partials or waits on a combine: one warp per (layer, sequence, head) segment when a wave of
   // resident warps holds them all (the wider pipeline shape first), else k consecutive whole
   // segments per warp, with the shape and k that put the fewest segments on the busiest SM.
-  // Otherwise the rows are split evenly over a full wave (stream-K), one layer per launch.
+  // Otherwise, over several layers whose segments are short beside a warp's share of the rows, whole
+  // segments cut by rows; else the rows are split evenly over a full wave (stream-K), one layer per
+  // launch.
   const int n_layers = a.n_layers < 1 ? 1 : a.n_layers;
   const int64_t nseg = (int64_t)n_layers * g.b * g.H;
   if (!decode_balanced(a)) {
-    if (n_layers > 1) return cudaErrorNotSupported;  // the caller launches the layers one by one
+    if (n_layers > 1) {
+      // Unbalanced segments over several layers: a wave of wide-pipeline warps takes whole segments
+      // cut by rows when the longest segment is at most 1/32 of a warp's even share (so no warp
+      // holds more than ~3 % above the mean); else the caller launches the layers one by one.
+      int occ_a = 0;
+      const cudaError_t e = decode_occupancy<T, D, AK, AS>(&occ_a);
+      if (e != cudaSuccess) return e;
+      int64_t NW = (int64_t)occ_a * num_sms;
+      if (NW > nseg) NW = nseg;
+      if (NW < 1 || 32 * a.max_segment > (int64_t)n_layers * a.R / NW) return cudaErrorNotSupported;
+      *plan = {4, (int)NW, AK * Lanes<D>::RPI, AS};
+      return launch_decode_cfg<T, D, AK, AS>(g, st, buf, a, NW, -1, stream, grid);
+    }
   } else {
     cudaError_t e;
     int occ_a = 0, occ_b = 0;

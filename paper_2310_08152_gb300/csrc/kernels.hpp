@@ -80,7 +80,7 @@ cudaError_t launch_compact(const Geometry& g, const Static& st, const Buffers& b
 
 struct DecodeArgs {
   int layer;             // the first layer of the launch
-  int n_layers = 1;      // layers layer .. layer + n_layers - 1 in one launch (balanced segments only)
+  int n_layers = 1;      // layers layer .. layer + n_layers - 1 in one launch (whole segments only)
   const DState* dstate;  // [b]
   const int64_t* P;      // [b+1] prefix sums of attended-range lengths (len - begin)
   int64_t R;             // H * P[b]
@@ -102,14 +102,16 @@ struct DecodeArgs {
 
 // How a decode launch split its work: mode 0 = stream-K over all rows, 1 / 2 = one warp per
 // (layer, sequence, head) segment with the wide / narrow pipeline, 3 = several consecutive whole
-// segments per warp; workers = warps; tile rows; stages.
+// segments per warp, 4 = consecutive whole segments per warp cut by rows (unbalanced segments over
+// several layers); workers = warps; tile rows; stages.
 struct DecodePlan {
   int mode, workers, tile_rows, stages;
 };
 
 // Returns the grid used through *grid (0 if nothing launched) and the plan through *plan.  A launch
-// over several layers (a.n_layers > 1) takes whole segments only: when the segments are not
-// balanced it launches nothing and returns cudaErrorNotSupported, and the caller goes layer by layer.
+// over several layers (a.n_layers > 1) takes whole segments only: when the longest segment is too
+// long beside a warp's share of the rows it launches nothing and returns cudaErrorNotSupported, and
+// the caller goes layer by layer.
 cudaError_t launch_decode(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a,
                           int num_sms, cudaStream_t stream, int* grid, DecodePlan* plan);
 

@@ -856,7 +856,7 @@ kvc_status kvc_decode_attention_layers(kvc_cache* c, int first, int n_layers, co
   st = c->ensure_cuda(stream);
   if (st != KVC_OK) return st;
   if (n_layers > 1) {
-    // balanced segments: every layer's in one launch (no per-launch prologue and drain per layer)
+    // whole segments: every layer's in one launch (no per-launch prologue and drain per layer)
     kvc::DecodeArgs a = decode_args(c, first, q, scale, out);
     a.n_layers = n_layers;
     a.q_layer_stride = q_layer_stride;
@@ -872,7 +872,7 @@ kvc_status kvc_decode_attention_layers(kvc_cache* c, int first, int n_layers, co
     }
     if (e != cudaErrorNotSupported) return cuda_fail(e, "decode kernel (layers)");
   }
-  // unbalanced segments (split over a wave of warps per layer): one launch per layer, in order
+  // segments too long to be taken whole (split over a wave of warps per layer): one launch per layer
   const uint16_t* qp = static_cast<const uint16_t*>(q);
   for (int i = 0; i < n_layers; ++i) {
     st = kvc_decode_attention(c, first + i, qp + i * q_layer_stride, scale, out + i * out_layer_stride, stream);

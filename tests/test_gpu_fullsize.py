@@ -117,6 +117,8 @@ def test_capacity_sweep_shapes_b4096_unbalanced_stream_k():
 def test_full_ragged():
     w = wl.ragged()
     run = _full(w, 32, check_at={0, 15, 31})
+    # the benchmark's launch configuration: every layer in one launch, whole segments cut by rows
+    assert run.cache.last_decode_plan["mode"] == 4, run.cache.last_decode_plan
     ln = run.cache.lengths()[0]
     assert ln.max() > 3000 and ln.min() < 400  # ragged: lengths span more than an order of magnitude
 

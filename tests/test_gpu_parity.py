@@ -417,3 +417,37 @@ def test_fused_layers_fall_back_to_per_layer_launches_when_unbalanced():
     for m in range(w.M):
         compare(o[m], ow.expected_decode(w, 2, m, [0, 1]), f"layer {m}")
     assert run.cache.device_status() == 0
+
+
+def test_fused_layers_whole_segments_cut_by_rows():
+    """Unbalanced (ragged) segments over many layers, each short beside a warp's even share of all the
+    layers' rows: one launch in which every warp takes a run of whole segments cut by rows (no split,
+    no combine).  Against the per-layer stream-K launches, which split segments and combine them, and
+    against the oracle on the first, a middle and the last layer."""
+    w = wl.ragged(b=64, lmin=64, lmax=700, M=24, steps=2)
+    run = harness.Runner(w, 2)
+    run.load_prompt()
+    inp = run.make_step_inputs(0)
+    run.append_only(inp)
+    rows = run.attended_rows()
+    assert rows.max() * w.b > 1.3 * rows.sum()  # unbalanced: the longest segment is above 1.3x the mean
+    one = torch.full((w.M, w.b, w.H, w.d), float("nan"), dtype=torch.float32, device="cuda")
+    for m in range(w.M):
+        kvc.kvc_decode_attention(run.cache.handle, m, inp.q[m], w.scale, one[m])
+    assert run.cache.last_decode_plan["mode"] == 0
+    l0 = run.cache.launch_count
+    many = run.cache.decode_attention_layers(inp.q, w.scale)
+    torch.cuda.synchronize()
+    plan = run.cache.last_decode_plan
+    assert run.cache.launch_count == l0 + 1
+    assert plan["mode"] == 4, plan
+    # the precondition of the plan: the longest segment within 1/32 of a warp's share of the rows
+    assert 32 * rows.max() <= w.M * w.H * rows.sum() // plan["workers"]
+    o, o1 = many.cpu().numpy(), one.cpu().numpy()
+    seqs = list(range(w.b))
+    for m in (0, w.M // 2, w.M - 1):
+        ref = ow.expected_decode(w, 1, m, seqs)
+        compare(o[m], ref, f"fused layer {m}")
+        compare(o1[m], ref, f"per-layer layer {m}")
+    compare(o.reshape(-1), o1.reshape(-1).astype(np.float64), "fused against per-layer, every layer")
+    assert run.cache.device_status() == 0
