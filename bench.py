@@ -102,8 +102,10 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(workload: str):
-    """DRAM bytes per decode launch from a committed ncu capture, if it was taken on this kernel source."""
+def recorded_traffic(workload: str, bytes_per_launch: float):
+    """DRAM bytes (read + write) per decode launch from a committed ncu capture taken on this kernel
+    source: the capture's DRAM bytes per algorithmic byte, scaled to this run's algorithmic bytes per
+    launch (the capture is a smaller case of the same plan; the ratio, not the size, carries over)."""
     p = os.path.join(ROOT, "profiles", "decode_traffic.json")
     try:
         with open(p) as f:
@@ -113,7 +115,7 @@ def recorded_traffic(workload: str):
     rec = j.get(workload)
     if not rec or rec.get("kernel_source_hash") != kernel_source_hash():
         return None
-    return rec.get("dram_bytes_per_launch")
+    return rec["dram_bytes_per_algorithmic_byte"] * bytes_per_launch
 
 
 class ClockSampler:
@@ -713,7 +715,7 @@ def run_kvc(args, w):
                          "frac": r["achieved"] / r["peak"], "frac_of_8tbs": r["achieved"] / 8000.0,
                          "peak_kind": r["peak_kind"],
                          "kernel": "decode_kernel (split-K single-query attention + log-sum-exp combine)",
-                         "traffic": recorded_traffic(w.name),
+                         "traffic": recorded_traffic(w.name, r["bytes"] / n_launch),
                          "bytes_per_launch_mean": r["bytes"] / n_launch,
                          "launch_us_mean": r["dec_total_s"] / n_launch * 1e6},
             "decode_plan": plan_record(r["plan"], r["dec_launches"] / args.steps),
