@@ -739,15 +739,16 @@ def run_kvc(args, w):
 
 
 def run_e2e(args, w, dev, world):
-    """The same steps through the public API with inputs in pinned host memory: each step copies its
-    token's K/V and the queries host->device and reads the outputs back device->host.  The timed
-    region runs `--e2e-reps` times, each on a fresh cache built from the same prompt, and the median
-    is reported with every sample: on a shared host a window's copies can stall."""
+    """The same steps through the public API with inputs in host memory: each step stages its token's
+    K/V and the queries into a pinned buffer, copies them host->device and reads the outputs back
+    device->host.  The timed region runs `--e2e-reps` times, each on a fresh cache built from the
+    same prompt, and the median is reported with every sample: on a shared host a window's copies
+    can stall."""
     vals, clocks = [], []
     h2d = d2h = 0
     for _ in range(max(1, args.e2e_reps)):
-        v, clk, h2d, d2h = _e2e_once(args, w, dev, world)
-        vals.append(v)
+        tokens, elapsed, clk, h2d, d2h = _e2e_once(args, w, dev, world)
+        vals.append(tokens / elapsed)
         if clk:
             clocks.append(clk)
     merged = None
@@ -769,12 +770,17 @@ def _e2e_once(args, w, dev, world):
     steps_total = args.warmup + args.steps
     run = harness.Runner(w, steps_total, device=dev)
     run.load_prompt()
+    # every step's inputs in ordinary (pageable) host memory, as a caller would hold them
     host_in = []
     for g in range(steps_total):
         inp = run.make_step_inputs(g)
-        host_in.append((inp.kinds, inp.kv_k.cpu().pin_memory(), inp.kv_v.cpu().pin_memory(),
-                        inp.q.cpu().pin_memory()))
+        host_in.append((inp.kinds, inp.kv_k.cpu(), inp.kv_v.cpu(), inp.q.cpu()))
     shape = (w.M, w.b, w.H, w.d)
+    # Two pinned staging sets: each step's inputs are copied into one on the host, then uploaded from
+    # it while the previous step computes; a set is refilled once its previous uploads have read it.
+    # (Uploading from a distinct pinned buffer per step -- 5 GB of pinned memory for the ragged
+    # workload -- made single 38 MB uploads take up to 9 ms and slowed the decodes they overlapped.)
+    stage = [tuple(torch.empty(shape, dtype=run.tdt).pin_memory() for _ in range(3)) for _ in range(2)]
     # Two sets of device inputs and outputs: an upload stream copies the next step's inputs while
     # the current step runs, and a download stream reads each step's outputs back while the next one
     # runs (one stream per direction, so the two copy engines never wait on each other).  Every
@@ -796,11 +802,14 @@ def _e2e_once(args, w, dev, world):
     def upload(g):
         i = g & 1
         kinds, hk, hv, hq = host_in[g]
+        ev_in[i].synchronize()  # the staging set's previous uploads have read it
+        for dst, src in zip(stage[i], (hk, hv, hq)):
+            dst.copy_(src)
         with torch.cuda.stream(up):
             up.wait_event(ev_done[i])   # the step that last used this set is done with its inputs
-            dk[i].copy_(hk, non_blocking=True)
-            dv[i].copy_(hv, non_blocking=True)
-            dq[i].copy_(hq, non_blocking=True)
+            dk[i].copy_(stage[i][0], non_blocking=True)
+            dv[i].copy_(stage[i][1], non_blocking=True)
+            dq[i].copy_(stage[i][2], non_blocking=True)
             ev_in[i].record(up)
 
     def one(g, last):
@@ -819,6 +828,7 @@ def _e2e_once(args, w, dev, world):
     for i in range(2):
         ev_done[i].record(comp)
         ev_out[i].record(comp)
+        ev_in[i].record(comp)
     upload(0)
     for g in range(args.warmup):
         one(g, g == args.warmup - 1)
@@ -828,7 +838,7 @@ def _e2e_once(args, w, dev, world):
     clocks = ClockSampler(dev.index)
     clocks.start()
     t0 = time.perf_counter()
-    upload(args.warmup)  # every timed step's inputs are uploaded inside the timed region
+    upload(args.warmup)  # every timed step's inputs are staged and uploaded inside the timed region
     for k in range(args.steps):
         one(args.warmup + k, k == args.steps - 1)
     torch.cuda.synchronize()
@@ -837,7 +847,7 @@ def _e2e_once(args, w, dev, world):
     tokens, elapsed = aggregate(w.b * args.steps, elapsed, dev)
     del run
     torch.cuda.empty_cache()
-    return tokens / elapsed, clk, h2d, d2h
+    return tokens, elapsed, clk, h2d, d2h
 
 
 def main():

@@ -451,3 +451,30 @@ def test_fused_layers_whole_segments_cut_by_rows():
         compare(o1[m], ref, f"per-layer layer {m}")
     compare(o.reshape(-1), o1.reshape(-1).astype(np.float64), "fused against per-layer, every layer")
     assert run.cache.device_status() == 0
+
+
+def test_local_attention_ragged_rings_fused_layers():
+    """Local Attention rings of different sizes over 24 layers (prompts of 64-700 tokens, window about
+    half the history, so every ring has wrapped): one decode launch in which warps take runs of whole
+    windows cut by rows, each window read in two parts around its ring's end.  Against the oracle's
+    Local Attention decode on the first, a middle and the last layer, two steps."""
+    base = wl.ragged(b=64, lmin=64, lmax=700, M=24, steps=3)
+    kinds = [np.zeros(int(n), np.uint8) for n in base.prompt_len]
+    w = dataclasses.replace(base, prompt_kinds=kinds, prompt_spans=[[] for _ in kinds], gen_kind=wl._normal_gen,
+                            name="ragged-local")
+    ratio = 0.5
+    r32 = float(np.float32(ratio))
+    run = harness.Runner(w, steps=3, policy=kvc.POLICY_LOCAL, local_ratio=ratio)
+    run.load_prompt()
+    out = torch.empty(w.M, w.b, w.H, w.d, dtype=torch.float32, device="cuda")
+    seqs = list(range(w.b))
+    for g in range(2):
+        l0 = run.cache.launch_count
+        run.step(run.make_step_inputs(g), out)
+        torch.cuda.synchronize()
+        assert run.cache.last_decode_plan["mode"] == 4, run.cache.last_decode_plan
+        assert run.cache.launch_count == l0 + 2  # the append and one decode launch
+        o = out.cpu().numpy()
+        for m in (0, w.M // 2, w.M - 1):
+            compare(o[m], ow.expected_local_decode(w, g + 1, m, seqs, r32), f"ragged local step {g} layer {m}")
+    assert run.cache.device_status() == 0
