@@ -458,15 +458,17 @@ struct Lanes {
   static_assert(D % 16 == 0 && CH % LPR == 0, "unsupported d_head");
 };
 
-// Shapes of the per-warp pipeline (rows per lane per tile x stages).  One warp per segment wants
-// the largest in-flight window that still lets every segment have a resident warp: 4x3 (64-row
-// tiles at d=64), else 2x3.  Stream-K runs a full wave of warps: 2x2 fits the most warps per SM.
-#ifndef KVC_DEC_SEG_KPT
-#define KVC_DEC_SEG_KPT 4
-#endif
-#ifndef KVC_DEC_SEG_STAGES
-#define KVC_DEC_SEG_STAGES 3
-#endif
+// Shapes of the per-warp pipeline (rows per lane per tile x stages).  Whole segments want the
+// largest in-flight window at three resident warps per SM, in as few tiles as possible (each tile
+// costs a fixed share of a warp's issue): 8x2 (128-row tiles, 64 KB per warp) at d=64, 6x2 (96-row
+// tiles, 60 KB) at d=80, 4x3 otherwise; measured on the full-size workloads against 4x3, 4x4 and
+// 6x3.  The narrow 2x3 shape fits the most warps when one warp per segment needs them.  Stream-K
+// runs a full wave of warps: 2x2 fits the most warps per SM.
+template <int D>
+struct WideShape {
+  static constexpr int KPT = D == 64 ? 8 : D == 80 ? 6 : 4;
+  static constexpr int S = (D == 64 || D == 80) ? 2 : 3;
+};
 #ifndef KVC_DEC_SEG2_KPT
 #define KVC_DEC_SEG2_KPT 2
 #endif
@@ -1059,12 +1061,12 @@ inline bool decode_balanced(const DecodeArgs& a) {
 template <typename T, int D>
 cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& buf, const DecodeArgs& a, int num_sms,
                             cudaStream_t stream, int* grid, DecodePlan* plan) {
-  constexpr int AK = KVC_DEC_SEG_KPT, AS = KVC_DEC_SEG_STAGES;
+  constexpr int AK = WideShape<D>::KPT, AS = WideShape<D>::S;
   constexpr int BK = KVC_DEC_SEG2_KPT, BS = KVC_DEC_SEG2_STAGES;
   constexpr int TK = KVC_DEC_STREAM_KPT, TS = KVC_DEC_STREAM_STAGES;
   // Balanced segments (longest within 1.3x of the mean) are never split, so no warp writes split-K
   // partials or waits on a combine: one warp per (layer, sequence, head) segment when a wave of
-  // resident warps holds them all (the wider pipeline shape first), else k consecutive whole
+  // resident warps holds them all (the wide pipeline shape first), else k consecutive whole
   // segments per warp, with the shape and k that put the fewest segments on the busiest SM.
   // Otherwise, over several layers whose segments are short beside a warp's share of the rows, whole
   // segments cut by rows; else the rows are split evenly over a full wave (stream-K), one layer per

@@ -212,7 +212,7 @@ def test_launch_counter_counts_kernels():
 
 def _mode_workloads():
     sms = torch.cuda.get_device_properties(0).multi_processor_count if torch.cuda.is_available() else 152
-    b_narrow = (5 * sms + 31) // 32  # more segments than one wave of the wide pipeline holds (4 warps/SM at d=64)
+    b_narrow = (5 * sms + 31) // 32  # more segments than one wave of the wide pipeline holds (3 warps/SM at d=64)
     # more segments than one wave of the narrow pipeline holds (8 warps/SM at d=64), and a count that
     # k does not divide, so the last worker takes fewer segments
     b_multi = (10 * sms + 31) // 32 + 1
