@@ -230,7 +230,7 @@ kvc_status kvc_decode_attention(kvc_cache* cache, int layer, const void* q, floa
  * kvc_decode_attention.  One launch covers every layer's segments, each (layer, sequence, head)
  * segment processed whole by one warp exactly as a per-layer launch with the same tile shape does it,
  * when the segments hold about as many rows as each other (the longest at most 1.3x the mean) or when
- * the longest is short beside a warp's even share of all the layers' rows (at most 1/32 of it; the
+ * the longest is short beside a warp's even share of all the layers' rows (at most 1/16 of it; the
  * warps then take runs of whole segments cut by rows).  Otherwise the layers are launched one by one,
  * in order, on `stream`, and on an error the layers before the failing one have been launched. */
 kvc_status kvc_decode_attention_layers(kvc_cache* cache, int first, int n_layers, const void* q, int64_t q_layer_stride,

@@ -1067,32 +1067,36 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
   // Balanced segments (longest within 1.3x of the mean) are never split, so no warp writes split-K
   // partials or waits on a combine: one warp per (layer, sequence, head) segment when a wave of
   // resident warps holds them all (the wide pipeline shape first), else k consecutive whole
-  // segments per warp, with the shape and k that put the fewest segments on the busiest SM.
-  // Otherwise, over several layers whose segments are short beside a warp's share of the rows, whole
-  // segments cut by rows; else the rows are split evenly over a full wave (stream-K), one layer per
-  // launch.
+  // segments per warp.  Otherwise, over several layers whose segments are short beside a warp's
+  // share of the rows, whole segments cut by rows; else the rows are split evenly over a full wave
+  // (stream-K), one layer per launch.  Whole segments shorter on average than six wide tiles go to
+  // the narrow shape (more warps per SM, less fixed work per tile and per segment): on ragged caches
+  // the wide shape wins from a mean of about 1,000 kept rows, the narrow one below about 500.
   const int n_layers = a.n_layers < 1 ? 1 : a.n_layers;
   const int64_t nseg = (int64_t)n_layers * g.b * g.H;
-  if (!decode_balanced(a)) {
-    if (n_layers > 1) {
-      // Unbalanced segments over several layers: a wave of wide-pipeline warps takes whole segments
-      // cut by rows when the longest segment is at most 1/32 of a warp's even share (so no warp
-      // holds more than ~3 % above the mean); else the caller launches the layers one by one.
-      int occ_a = 0;
-      const cudaError_t e = decode_occupancy<T, D, AK, AS>(&occ_a);
-      if (e != cudaSuccess) return e;
-      int64_t NW = (int64_t)occ_a * num_sms;
-      if (NW > nseg) NW = nseg;
-      if (NW < 1 || 32 * a.max_segment > (int64_t)n_layers * a.R / NW) return cudaErrorNotSupported;
-      *plan = {4, (int)NW, AK * Lanes<D>::RPI, AS};
-      return launch_decode_cfg<T, D, AK, AS>(g, st, buf, a, NW, -1, stream, grid);
-    }
-  } else {
+  const bool short_segs = a.n_segments > 0 && a.R < 6 * (int64_t)(AK * Lanes<D>::RPI) * a.n_segments;
+  const bool balanced = decode_balanced(a);
+  if (balanced || n_layers > 1) {
     cudaError_t e;
     int occ_a = 0, occ_b = 0;
     e = decode_occupancy<T, D, AK, AS>(&occ_a);
     if (e == cudaSuccess) e = decode_occupancy<T, D, BK, BS>(&occ_b);
     if (e != cudaSuccess) return e;
+    if (!balanced) {
+      // Unbalanced segments over several layers: a wave of warps takes whole segments cut by rows
+      // when the longest segment is at most 1/16 of a warp's even share (so no warp holds more than
+      // ~6 % above the mean); else the caller launches the layers one by one.
+      const int occ = short_segs ? occ_b : occ_a;
+      int64_t NW = (int64_t)occ * num_sms;
+      if (NW > nseg) NW = nseg;
+      if (NW < 1 || 16 * a.max_segment > (int64_t)n_layers * a.R / NW) return cudaErrorNotSupported;
+      if (short_segs) {
+        *plan = {4, (int)NW, BK * Lanes<D>::RPI, BS};
+        return launch_decode_cfg<T, D, BK, BS>(g, st, buf, a, NW, -1, stream, grid);
+      }
+      *plan = {4, (int)NW, AK * Lanes<D>::RPI, AS};
+      return launch_decode_cfg<T, D, AK, AS>(g, st, buf, a, NW, -1, stream, grid);
+    }
     if (nseg <= (int64_t)occ_a * num_sms) {
       *plan = {1, (int)nseg, AK * Lanes<D>::RPI, AS};
       return launch_decode_cfg<T, D, AK, AS>(g, st, buf, a, nseg, 1, stream, grid);
@@ -1101,8 +1105,10 @@ cudaError_t launch_decode_t(const Geometry& g, const Static& st, const Buffers& 
       *plan = {2, (int)nseg, BK * Lanes<D>::RPI, BS};
       return launch_decode_cfg<T, D, BK, BS>(g, st, buf, a, nseg, 1, stream, grid);
     }
+    // several whole segments per warp: the narrow shape for short segments, else the shape and k that
+    // put the fewest segments on the busiest SM
     const SegSplit sa = seg_split(nseg, occ_a, num_sms), sb = seg_split(nseg, occ_b, num_sms);
-    if (sa.busiest <= sb.busiest) {
+    if (!short_segs && sa.busiest <= sb.busiest) {
       *plan = {3, (int)sa.workers, AK * Lanes<D>::RPI, AS};
       return launch_decode_cfg<T, D, AK, AS>(g, st, buf, a, sa.workers, sa.k, stream, grid);
     }
