@@ -17,6 +17,7 @@ shards by sequence with no exchange); value = tokens of all ranks / max time ove
 from __future__ import annotations
 
 import argparse
+import collections
 import dataclasses
 import hashlib
 import json
@@ -579,6 +580,7 @@ def timed_decode_steps(run, w, inputs, warmup: int, steps: int, world: int = 1, 
     ones = np.ones(w.b, np.int32)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
     bytes_per_step, dec_launches = [], 0
+    plans = collections.Counter()  # the plan each step's decode used (mode, warps, tile rows, stages)
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         dist.barrier()
@@ -600,6 +602,7 @@ def timed_decode_steps(run, w, inputs, warmup: int, steps: int, world: int = 1, 
         if rc:
             raise kvc.KvcError(rc, kvc.lib().kvc_last_error().decode())
         dec_launches += run.cache.launch_count - l0
+        plans[tuple(run.cache.last_decode_plan.values())] += 1
         seq, cl, cr = run.step_spans(inp.kinds)
         run.g += 1
         if seq:
@@ -613,7 +616,9 @@ def timed_decode_steps(run, w, inputs, warmup: int, steps: int, world: int = 1, 
     dec_total_s = sum(dec_us) / 1e6
     achieved = sum(bytes_per_step) / dec_total_s / 1e9
     peak, peak_kind = measured_hbm_peak()
-    plan = run.cache.last_decode_plan
+    common, n_common = plans.most_common(1)[0]
+    plan = dict(zip(("mode", "workers", "tile_rows", "stages"), common))
+    plan["share_of_steps"] = n_common / steps
     return {"elapsed": elapsed, "tokens": w.b * steps, "launches": launches, "dec_launches": dec_launches,
             "dec_total_s": dec_total_s, "dec_us": dec_us, "bytes": sum(bytes_per_step), "achieved": achieved,
             "peak": peak, "peak_kind": peak_kind, "plan": plan, "clocks": clk}
@@ -625,7 +630,8 @@ PLAN_NAMES = ["stream-K", "warp per segment (wide)", "warp per segment (narrow)"
 
 def plan_record(plan, launches_per_step: float):
     return {"mode": PLAN_NAMES[plan["mode"]] if plan["mode"] >= 0 else None, "warps": plan["workers"],
-            "tile_rows": plan["tile_rows"], "stages": plan["stages"], "launches_per_step": launches_per_step}
+            "tile_rows": plan["tile_rows"], "stages": plan["stages"], "launches_per_step": launches_per_step,
+            "share_of_steps": plan.get("share_of_steps")}
 
 
 def measure_workload(name: str, dev, steps: int, warmup: int = 3):
