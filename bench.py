@@ -720,7 +720,7 @@ def run_kvc(args, w):
             "roofline": {"bound": "hbm", "achieved": r["achieved"], "peak": r["peak"], "unit": "GB/s",
                          "frac": r["achieved"] / r["peak"], "frac_of_8tbs": r["achieved"] / 8000.0,
                          "peak_kind": r["peak_kind"],
-                         "kernel": "decode_kernel (split-K single-query attention + log-sum-exp combine)",
+                         "kernel": "decode_kernel (single-query attention over the kept rows: whole segments per warp, or split-K with a log-sum-exp combine)",
                          "traffic": recorded_traffic(w.name, r["bytes"] / n_launch),
                          "bytes_per_launch_mean": r["bytes"] / n_launch,
                          "launch_us_mean": r["dec_total_s"] / n_launch * 1e6},
