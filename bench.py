@@ -653,6 +653,7 @@ def measure_workload(name: str, dev, steps: int, warmup: int = 3):
     torch.cuda.empty_cache()
     n_launch = max(1, r["dec_launches"])
     return {"workload": name, "tokens_per_s": r["tokens"] / r["elapsed"], "steps": steps,
+            "decode_attention_tokens_per_s": r["tokens"] / r["dec_total_s"],
             "decode": {"achieved": r["achieved"], "peak": r["peak"], "unit": "GB/s",
                        "frac": r["achieved"] / r["peak"], "frac_of_8tbs": r["achieved"] / 8000.0,
                        "peak_kind": r["peak_kind"], "bytes_per_launch_mean": r["bytes"] / n_launch,
@@ -727,6 +728,8 @@ def run_kvc(args, w):
             "decode_plan": plan_record(r["plan"], r["dec_launches"] / args.steps),
             "decode_us_per_step": {"min": dec_us[0], "median": statistics.median(dec_us), "max": dec_us[-1]},
             "decode_share_of_step": r["dec_total_s"] / r["elapsed"],
+            # b / (decode kernel time per step), the decode-attention rate alone; `value` is per whole step
+            "decode_attention_tokens_per_s": r["tokens"] / r["dec_total_s"],
             "compaction": compaction,
             "prompt_write_time_freeing": prompt_free,
             "prefill": prefill,
