@@ -21,7 +21,6 @@ import collections
 import dataclasses
 import hashlib
 import json
-import math
 import os
 import statistics
 import subprocess
